@@ -1,0 +1,151 @@
+"""Cycle-by-cycle stepper for tiny tile graphs (TEST INFRASTRUCTURE ONLY).
+
+A second, independent statement of the scheduling definition (Section 5.1 to
+5.3) used to pin the C oracle on tiny inputs.  It differs from the oracle on
+purpose in everything but the definition:
+
+* time advances one cycle at a time (t = 0, 1, 2, ...), no event skipping;
+* nothing is tracked incrementally: readiness, warp heads, resource usage and
+  CTA residency are recomputed from the partial schedule at every decision;
+* a resource class is free at t when fewer than ``cap`` of the nodes already
+  started on it satisfy start <= t < start + occupancy (counting, not the
+  server free-time multiset the oracle keeps).
+
+Pure Python; only for graphs of a few dozen nodes with short latencies.
+"""
+from __future__ import annotations
+
+LOAD, SMEM, MMA, EW, STORE, BAR, NOP = range(7)
+ISSUE = 1
+
+
+def node_costs(ty, work, lat_extra, prm):
+    """(per-SM class or None, its occupancy, HBM occupancy or None, latency)."""
+    def cdiv(a, b):
+        return -(-a // b)
+    num = {"hbm": prm[2], "tma": prm[4], "smem": prm[6], "mma": prm[8], "alu": prm[10]}
+    if ty == LOAD:
+        cls, occ, hocc, base = "tma", cdiv(work, num["tma"]), cdiv(work, num["hbm"]), prm[5] + prm[3]
+    elif ty == STORE:
+        cls, occ, hocc, base = "tma", cdiv(work, num["tma"]), cdiv(work, num["hbm"]), prm[5]
+    elif ty == SMEM:
+        cls, occ, hocc, base = "lsu", cdiv(work, num["smem"]), None, prm[7]
+    elif ty == MMA:
+        cls, occ, hocc, base = "tensor", cdiv(work, num["mma"]), None, prm[9]
+    elif ty == EW:
+        cls, occ, hocc, base = "alu", cdiv(work, num["alu"]), None, prm[11]
+    elif ty == BAR:
+        cls, occ, hocc, base = "bar", 1, None, prm[12]
+    else:
+        cls, occ, hocc, base = None, 0, None, 0
+    lat = base + lat_extra + max([0] + ([occ] if cls else []) + ([hocc] if hocc is not None else []))
+    return cls, occ, hocc, lat
+
+
+def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel, warps_per_cta, prm,
+             t_limit=None):
+    """Returns (status, makespan, start list, finish list, cta_sm list).
+
+    status: 0 ok, -6 a finish above 2^31-1, -8 no progress possible.
+    """
+    n = len(type_)
+    C = len(cta_kernel)
+    prm = [int(x) for x in prm]
+    num_sms, cps = prm[0], prm[1]
+    cap = {"tensor": prm[13], "tma": prm[14], "lsu": prm[15], "alu": prm[16], "bar": prm[17]}
+    cap_hbm = prm[18]
+    costs = [node_costs(int(type_[v]), int(work[v]), int(lat_extra[v]), prm) for v in range(n)]
+    preds = [[] for _ in range(n)]
+    for u in range(n):
+        for e in range(int(row_ptr[u]), int(row_ptr[u + 1])):
+            preds[int(col[e])].append((u, int(ekind[e])))
+    members = [[v for v in range(n) if int(cta[v]) == c] for c in range(C)]
+    start = [None] * n
+    cta_sm = [-1] * C
+    launched = [False] * C
+    total_lat = sum(c[3] for c in costs)
+    if t_limit is None:
+        t_limit = total_lat + 2
+
+    def finish(v):
+        return start[v] + costs[v][3]
+
+    def retired(c, t):
+        return launched[c] and all(start[v] is not None and finish(v) <= t for v in members[c])
+
+    def is_head(v):
+        return all(start[u] is not None for u in members[int(cta[v])]
+                   if u < v and int(warp[u]) == int(warp[v]))
+
+    def busy(cls, sm, t):
+        k = 0
+        for u in range(n):
+            if start[u] is None or costs[u][0] != cls or cta_sm[int(cta[u])] != sm:
+                continue
+            if start[u] <= t < start[u] + costs[u][1]:
+                k += 1
+        return k
+
+    def busy_hbm(t):
+        return sum(1 for u in range(n) if start[u] is not None and costs[u][2] is not None
+                   and start[u] <= t < start[u] + costs[u][2])
+
+    def issuable(v, t):
+        c = int(cta[v])
+        if start[v] is not None or not launched[c] or not is_head(v):
+            return False
+        rel = 0
+        for u, k in preds[v]:
+            if start[u] is None:
+                return False
+            rel = max(rel, start[u] if k == ISSUE else finish(u))
+        if rel > t:
+            return False
+        cls, _occ, hocc, _lat = costs[v]
+        if cls is not None and busy(cls, cta_sm[c], t) >= cap[cls]:
+            return False
+        if hocc is not None and busy_hbm(t) >= cap_hbm:
+            return False
+        return True
+
+    t = 0
+    while True:
+        changed = True
+        while changed:
+            changed = False
+            # CTA launches in ascending order, each on the lowest SM with a free slot
+            while True:
+                c = sum(launched)
+                if c >= C:
+                    break
+                if any(int(cta_kernel[d]) < int(cta_kernel[c]) and not retired(d, t) for d in range(c)):
+                    break
+                occupied = [0] * num_sms
+                for d in range(c):
+                    if not retired(d, t):
+                        occupied[cta_sm[d]] += 1
+                free = [s for s in range(num_sms) if occupied[s] < cps]
+                if not free:
+                    break
+                launched[c] = True
+                cta_sm[c] = free[0]
+                changed = True
+            cands = [v for v in range(n) if issuable(v, t)]
+            if cands:
+                v = min(cands)
+                start[v] = t
+                if finish(v) > 2**31 - 1:
+                    return -6, 0, start, [None] * n, cta_sm
+                changed = True
+        if all(s is not None for s in start):
+            fin = [finish(v) for v in range(n)]
+            return 0, max(fin, default=0), start, fin, cta_sm
+        t += 1
+        if t > t_limit:
+            return -8, 0, start, [None] * n, cta_sm
+
+
+def simulate_graph(g, prm, **kw):
+    """Same, for a single workloads.Graph."""
+    return simulate(g.row_ptr, g.col, g.ekind, g.type, g.warp, g.cta, g.work, g.lat_extra, g.cta_kernel,
+                    g.warps_per_cta, prm, **kw)
