@@ -1,0 +1,214 @@
+/*
+ * gts.h -- C ABI of libgts, a batched graph-driven tile-graph simulator for
+ * sm_103a (GB300).
+ *
+ * The library computes what the graph-driven simulation backend of
+ * GPU-Tile-Sim computes (Section 5): given a warp-centric tile graph
+ * G = (V, E) (Section 4.1) and a hardware description, the start and finish
+ * cycle of every node and the kernel makespan.  It does so for many
+ * independent hardware/tiling design points in one launch, one design point
+ * per warp.
+ *
+ * Semantics (Section 5.1 execution flow, Section 5.2 throughput models,
+ * Section 5.3 runtime control), with the framework's fixed readings:
+ *  - each logical warp issues its nodes in program order (ascending id);
+ *  - a DATA edge u->v releases v when u completes, an ISSUE (order) edge when
+ *    u issues, in the same cycle;
+ *  - a node of type LOAD/STORE takes one TMA server of its SM and one of the
+ *    global HBM servers, SMEM one LSU server, MMA one TENSOR server, EW one
+ *    ALU server, BAR one BAR server, NOP none; each for its occupancy
+ *    ceil(work / rate) cycles (BAR: 1 cycle); the node's latency is
+ *    L = base(type) + lat_extra + max occupancy, and finish = start + L;
+ *  - CTAs launch in ascending id, each on the lowest SM with a free slot,
+ *    at the cycle a slot frees; a CTA retires when all its nodes completed;
+ *    a CTA of kernel k launches only after every CTA of kernels < k retired;
+ *  - at every cycle the scheduler issues, one at a time, the lowest node id
+ *    among warp heads whose predecessors are released and whose units have a
+ *    free server, launching CTAs first, until nothing changes; then it moves to
+ *    the next event cycle.
+ *  Cycles are int32; a finish above 2^31-1 is reported as GTS_ERR_OVERFLOW.
+ *
+ * Conventions:
+ *  - Every pointer named d_* or held in gts_graph_desc is a DEVICE pointer on
+ *    the current CUDA device, owned by the caller; h_* pointers are host
+ *    pointers.  The library never allocates device memory: the caller supplies
+ *    the graph workspace and the simulation scratch, sized by the *_bytes()
+ *    queries.  Handles borrow the caller's buffers and must not outlive them.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *    Calls enqueue work on it and return without waiting, except
+ *    gts_graph_create, gts_params_upload and gts_read_results, which wait for
+ *    the stream.
+ *  - Host-side errors are returned as a status; gts_last_error() then holds a
+ *    message for the calling thread.  Per-design-point errors (bad parameter
+ *    row, overflow, deadlock, step limit) are written to d_status[p]; the other
+ *    points are still simulated.  No call throws, traps or spins without bound.
+ */
+#ifndef GTS_H
+#define GTS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t gts_status;
+#define GTS_OK                  0
+#define GTS_ERR_INVALID_ARG    (-1)  /* null pointer, size out of range, bad flags */
+#define GTS_ERR_INVALID_GRAPH  (-2)  /* graph breaks the contract below */
+#define GTS_ERR_INVALID_PARAMS (-3)  /* parameter row: rate/cap/count < 1, latency < 0, bad graph index */
+#define GTS_ERR_CUDA           (-4)  /* a CUDA runtime call failed */
+#define GTS_ERR_NOMEM          (-5)  /* workspace or scratch smaller than required */
+#define GTS_ERR_OVERFLOW       (-6)  /* some finish cycle exceeds 2^31-1 (per point) */
+#define GTS_ERR_STEP_LIMIT     (-7)  /* per-point loop bound reached (never for valid input) */
+#define GTS_ERR_DEADLOCK       (-8)  /* no event left while nodes remain (per point) */
+#define GTS_ERR_UNSUPPORTED    (-9)  /* row needs more on-chip state than one warp may hold */
+
+/* Node operation types (Section 4.1 operation descriptor). */
+#define GTS_LOAD  0   /* global/TMA -> shared; work = bytes; TMA + HBM; base tma_lat + dram_lat */
+#define GTS_SMEM  1   /* shared <-> registers; work = bytes; LSU; base smem_lat */
+#define GTS_MMA   2   /* tensor-core MMA; work = FMAs; TENSOR; base mma_lat */
+#define GTS_EW    3   /* elementwise / softmax / norm; work = ops; ALU; base alu_lat */
+#define GTS_STORE 4   /* shared/registers -> global; work = bytes; TMA + HBM; base tma_lat */
+#define GTS_BAR   5   /* mbarrier / named-barrier wait; BAR for 1 cycle; base bar_lat */
+#define GTS_NOP   6   /* pure synchronisation point; no unit; base 0 */
+
+/* Edge kinds (Section 4.1 data and order edges). */
+#define GTS_EDGE_DATA  0  /* released when the producer completes */
+#define GTS_EDGE_ISSUE 1  /* released when the producer issues */
+
+/* Parameter row: GTS_NPARAM int32 per design point (Table "GPU configurations"
+ * quantities in cycles and bytes/FMAs/ops per cycle). */
+#define GTS_NPARAM 24
+#define GTS_P_NUM_SMS      0
+#define GTS_P_CTAS_PER_SM  1
+#define GTS_P_HBM_BPC      2   /* global DRAM bytes per cycle (one HBM server) */
+#define GTS_P_DRAM_LAT     3
+#define GTS_P_TMA_BPC      4
+#define GTS_P_TMA_LAT      5
+#define GTS_P_SMEM_BPC     6
+#define GTS_P_SMEM_LAT     7
+#define GTS_P_MMA_FMA_PC   8
+#define GTS_P_MMA_LAT      9
+#define GTS_P_ALU_OPS_PC  10
+#define GTS_P_ALU_LAT     11
+#define GTS_P_BAR_LAT     12
+#define GTS_P_CAP_TENSOR  13   /* servers per SM */
+#define GTS_P_CAP_TMA     14
+#define GTS_P_CAP_LSU     15
+#define GTS_P_CAP_ALU     16
+#define GTS_P_CAP_BAR     17
+#define GTS_P_CAP_HBM     18   /* global HBM servers */
+#define GTS_P_GRAPH_INDEX 19   /* which graph of a stacked set this point runs */
+/* 20..23 reserved, must be 0 */
+
+/* Flags of gts_simulate_batch. */
+#define GTS_FULL_TRACE  1u  /* write d_start / d_finish [n_points][row_nodes] */
+#define GTS_WANT_DIGEST 2u  /* write d_digest[n_points] */
+#define GTS_WANT_CTA_SM 4u  /* write d_cta_sm [n_points][row_ctas] (-1: never launched) */
+
+typedef struct gts_graph gts_graph;
+typedef struct gts_params gts_params;
+typedef struct gts_results gts_results;
+
+/*
+ * A tile graph, or a stack of n_graphs independent tile graphs (Section 4.1).
+ * Ids are global over the stack; graph g owns nodes graph_node_off[g] ..
+ * graph_node_off[g+1]-1 and CTAs graph_cta_off[g] .. graph_cta_off[g+1]-1.
+ * Contract (checked by gts_graph_create, else GTS_ERR_INVALID_GRAPH):
+ *  - successors are CSR: row_ptr[0] = 0, row_ptr non-decreasing,
+ *    row_ptr[n_nodes] = n_edges; col[e] is the successor, ekind[e] its kind;
+ *  - every edge u->v has u < v and stays inside its graph (ids are a
+ *    topological order);
+ *  - type < 7, warp < warps_per_cta, cta inside the node's graph;
+ *  - cta_kernel is non-decreasing within each graph.
+ * The program order of each (cta, warp) stream is ascending id.
+ * Limits: n_nodes < 2^31, n_ctas < 2^24, warps_per_cta <= 128.
+ */
+typedef struct {
+  uint32_t n_nodes, n_edges, n_ctas, warps_per_cta, n_graphs;
+  const uint32_t *graph_node_off;   /* [n_graphs+1]; NULL allowed when n_graphs == 1 */
+  const uint32_t *graph_cta_off;    /* [n_graphs+1]; NULL allowed when n_graphs == 1 */
+  const uint32_t *row_ptr;          /* [n_nodes+1] */
+  const uint32_t *col;              /* [n_edges] */
+  const uint8_t  *ekind;            /* [n_edges] GTS_EDGE_* */
+  const uint8_t  *type;             /* [n_nodes] GTS_LOAD.. */
+  const uint16_t *warp;             /* [n_nodes] CTA-local logical warp */
+  const uint32_t *cta;              /* [n_nodes] */
+  const uint32_t *work;             /* [n_nodes] bytes / FMAs / ops */
+  const uint32_t *lat_extra;        /* [n_nodes] extra latency, cycles */
+  const uint32_t *cta_kernel;       /* [n_ctas] */
+  void *workspace;                  /* device, >= gts_graph_workspace_bytes(...) */
+  size_t workspace_bytes;
+} gts_graph_desc;
+
+/* Bytes of device workspace gts_graph_create needs for a graph of this size
+ * (packed node records, successor and predecessor lists, stream heads).
+ * Returns 0 when a size is out of range. */
+size_t gts_graph_workspace_bytes(uint32_t n_nodes, uint32_t n_edges, uint32_t n_ctas,
+                                 uint32_t warps_per_cta, uint32_t n_graphs);
+
+/* Checks the graph contract and builds the derived device arrays into
+ * desc->workspace (Section 4.1 graph, Section 5.1 per-TB streams).  Copies the
+ * graph to the host to check and pack it, then back; waits for `stream`.
+ * *out borrows desc->cta_kernel and desc->workspace.
+ * Errors: INVALID_ARG, INVALID_GRAPH (message names the first offending
+ * index), NOMEM (workspace too small), CUDA. */
+gts_status gts_graph_create(const gts_graph_desc *desc, void *stream, gts_graph **out);
+gts_status gts_graph_destroy(gts_graph *graph);
+
+/* Registers a table of design points: d_params is [n_points][GTS_NPARAM]
+ * int32 on the device, borrowed by *out.  Copies it to the host to size the
+ * per-warp on-chip state of each row; waits for `stream`.  Rows that break the
+ * parameter rules are not an error here: gts_simulate_batch reports them as
+ * GTS_ERR_INVALID_PARAMS in d_status.  Errors: INVALID_ARG, CUDA. */
+gts_status gts_params_upload(gts_graph *graph, const int32_t *d_params, uint32_t n_points,
+                             void *stream, gts_params **out);
+gts_status gts_params_destroy(gts_params *params);
+
+/* Per-point output row lengths: start/finish rows hold gts_row_nodes() entries
+ * (the largest graph of the stack), cta_sm rows gts_row_ctas(). */
+uint32_t gts_row_nodes(const gts_graph *graph);
+uint32_t gts_row_ctas(const gts_graph *graph);
+
+/* Device scratch gts_simulate_batch wants for `flags`: without GTS_FULL_TRACE
+ * the per-warp start/finish rows live in scratch; with it, none is needed.
+ * Returns the size that lets every resident warp work; a smaller non-zero
+ * scratch runs fewer design points at a time. */
+size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint32_t flags);
+
+/*
+ * Simulates design points first_point .. first_point+n_points-1 of `params`
+ * on `graph`.  Output arrays are indexed by q = p - first_point:
+ *   d_makespan[q], d_status[q]                      (required)
+ *   d_start[q*row_nodes + v], d_finish[...]         (GTS_FULL_TRACE; graph-local v)
+ *   d_digest[q]                                     (GTS_WANT_DIGEST)
+ *   d_cta_sm[q*row_ctas + c]                        (GTS_WANT_CTA_SM; graph-local c)
+ * Start/finish/digest/cta_sm of a point whose status is not GTS_OK are
+ * unspecified.  The digest is sum over v of splitmix64-finalise(
+ * (v << 32 | (uint32)start) ^ ((uint64)(uint32)finish * 0x9E3779B97F4A7C15)) mod 2^64.
+ * Enqueues on `stream` and returns; *out (may be NULL) remembers the arrays
+ * for gts_read_results.  Errors: INVALID_ARG, NOMEM (scratch too small), CUDA.
+ */
+gts_status gts_simulate_batch(gts_graph *graph, gts_params *params,
+                              uint32_t first_point, uint32_t n_points, uint32_t flags,
+                              int32_t *d_start, int32_t *d_finish,
+                              int32_t *d_makespan, int32_t *d_status,
+                              uint64_t *d_digest, int32_t *d_cta_sm,
+                              void *d_scratch, size_t scratch_bytes,
+                              void *stream, gts_results **out);
+
+/* Waits for the batch and copies its per-point arrays to the host (any h_*
+ * may be NULL; n_points <= the batch's).  Errors: INVALID_ARG, CUDA. */
+gts_status gts_read_results(gts_results *results, int32_t *h_makespan, int32_t *h_status,
+                            uint64_t *h_digest, uint32_t n_points);
+gts_status gts_results_destroy(gts_results *results);
+
+/* Message for the calling thread's last non-OK host-side status ("" if none). */
+const char *gts_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GTS_H */

@@ -1,0 +1,283 @@
+"""Python binding of libgts (argument marshalling only).
+
+Functions named like the C ABI in include/gts.h take plain integers (device
+pointers, sizes, stream handles) and return handles or raise ``GtsError``.
+``DeviceGraph`` / ``DeviceParams`` / ``simulate`` add torch-owned device
+buffers around them: torch supplies device memory and streams, every step of
+the simulation runs in libgts's CUDA kernels.  There is no CPU fallback: if
+libgts is not built, importing works but every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_build", "libgts.so")
+
+GTS_OK = 0
+GTS_ERR_INVALID_ARG = -1
+GTS_ERR_INVALID_GRAPH = -2
+GTS_ERR_INVALID_PARAMS = -3
+GTS_ERR_CUDA = -4
+GTS_ERR_NOMEM = -5
+GTS_ERR_OVERFLOW = -6
+GTS_ERR_STEP_LIMIT = -7
+GTS_ERR_DEADLOCK = -8
+GTS_ERR_UNSUPPORTED = -9
+
+GTS_FULL_TRACE = 1
+GTS_WANT_DIGEST = 2
+GTS_WANT_CTA_SM = 4
+
+EXPORTS = ("gts_graph_workspace_bytes", "gts_graph_create", "gts_graph_destroy", "gts_params_upload",
+           "gts_params_destroy", "gts_row_nodes", "gts_row_ctas", "gts_scratch_bytes", "gts_simulate_batch",
+           "gts_read_results", "gts_results_destroy", "gts_last_error")
+
+
+class GtsError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"libgts status {status}: {msg}")
+        self.status = status
+
+
+class GraphDesc(ctypes.Structure):
+    _fields_ = [("n_nodes", ctypes.c_uint32), ("n_edges", ctypes.c_uint32), ("n_ctas", ctypes.c_uint32),
+                ("warps_per_cta", ctypes.c_uint32), ("n_graphs", ctypes.c_uint32),
+                ("graph_node_off", ctypes.c_void_p), ("graph_cta_off", ctypes.c_void_p),
+                ("row_ptr", ctypes.c_void_p), ("col", ctypes.c_void_p), ("ekind", ctypes.c_void_p),
+                ("type", ctypes.c_void_p), ("warp", ctypes.c_void_p), ("cta", ctypes.c_void_p),
+                ("work", ctypes.c_void_p), ("lat_extra", ctypes.c_void_p), ("cta_kernel", ctypes.c_void_p),
+                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t)]
+
+
+_lib = None
+
+
+def load():
+    """The loaded libgts (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"libgts is not built ({LIB_PATH}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, u32, i32, sz = ctypes.c_void_p, ctypes.c_uint32, ctypes.c_int32, ctypes.c_size_t
+    pp = ctypes.POINTER(ctypes.c_void_p)
+    lib.gts_graph_workspace_bytes.argtypes = [u32, u32, u32, u32, u32]
+    lib.gts_graph_workspace_bytes.restype = sz
+    lib.gts_graph_create.argtypes = [ctypes.POINTER(GraphDesc), vp, pp]
+    lib.gts_graph_create.restype = i32
+    lib.gts_graph_destroy.argtypes = [vp]
+    lib.gts_graph_destroy.restype = i32
+    lib.gts_params_upload.argtypes = [vp, vp, u32, vp, pp]
+    lib.gts_params_upload.restype = i32
+    lib.gts_params_destroy.argtypes = [vp]
+    lib.gts_params_destroy.restype = i32
+    lib.gts_row_nodes.argtypes = [vp]
+    lib.gts_row_nodes.restype = u32
+    lib.gts_row_ctas.argtypes = [vp]
+    lib.gts_row_ctas.restype = u32
+    lib.gts_scratch_bytes.argtypes = [vp, vp, u32]
+    lib.gts_scratch_bytes.restype = sz
+    lib.gts_simulate_batch.argtypes = [vp, vp, u32, u32, u32, vp, vp, vp, vp, vp, vp, vp, sz, vp, pp]
+    lib.gts_simulate_batch.restype = i32
+    lib.gts_read_results.argtypes = [vp, vp, vp, vp, u32]
+    lib.gts_read_results.restype = i32
+    lib.gts_results_destroy.argtypes = [vp]
+    lib.gts_results_destroy.restype = i32
+    lib.gts_last_error.argtypes = []
+    lib.gts_last_error.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+def _check(status):
+    if status != GTS_OK:
+        raise GtsError(status, load().gts_last_error().decode())
+
+
+# ---------------------------------------------------------------- raw ABI (same names)
+def gts_graph_workspace_bytes(n_nodes, n_edges, n_ctas, warps_per_cta, n_graphs):
+    return int(load().gts_graph_workspace_bytes(n_nodes, n_edges, n_ctas, warps_per_cta, n_graphs))
+
+
+def gts_graph_create(desc: GraphDesc, stream: int = 0):
+    h = ctypes.c_void_p()
+    _check(load().gts_graph_create(ctypes.byref(desc), stream, ctypes.byref(h)))
+    return h.value
+
+
+def gts_graph_destroy(graph):
+    _check(load().gts_graph_destroy(graph))
+
+
+def gts_params_upload(graph, d_params: int, n_points: int, stream: int = 0):
+    h = ctypes.c_void_p()
+    _check(load().gts_params_upload(graph, d_params, n_points, stream, ctypes.byref(h)))
+    return h.value
+
+
+def gts_params_destroy(params):
+    _check(load().gts_params_destroy(params))
+
+
+def gts_row_nodes(graph):
+    return int(load().gts_row_nodes(graph))
+
+
+def gts_row_ctas(graph):
+    return int(load().gts_row_ctas(graph))
+
+
+def gts_scratch_bytes(graph, params, flags):
+    return int(load().gts_scratch_bytes(graph, params, flags))
+
+
+def gts_simulate_batch(graph, params, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status,
+                       d_digest, d_cta_sm, d_scratch, scratch_bytes, stream=0, want_handle=False):
+    h = ctypes.c_void_p()
+    _check(load().gts_simulate_batch(graph, params, first_point, n_points, flags, d_start, d_finish, d_makespan,
+                                     d_status, d_digest, d_cta_sm, d_scratch, scratch_bytes, stream,
+                                     ctypes.byref(h) if want_handle else None))
+    return h.value if want_handle else None
+
+
+def gts_read_results(results, h_makespan, h_status, h_digest, n_points):
+    _check(load().gts_read_results(results, h_makespan, h_status, h_digest, n_points))
+
+
+def gts_results_destroy(results):
+    _check(load().gts_results_destroy(results))
+
+
+def gts_last_error():
+    return load().gts_last_error().decode()
+
+
+# ---------------------------------------------------------------- torch-owned buffers
+def _stream_handle(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+class DeviceGraph:
+    """A workloads.Graph resident on the GPU, validated and packed by libgts."""
+
+    def __init__(self, graph, device="cuda", stream=None):
+        import torch
+        self.graph = graph
+        dev = torch.device(device)
+
+        def t(a):
+            a = np.ascontiguousarray(a)
+            if a.dtype == np.uint32:
+                a = a.view(np.int32)
+            elif a.dtype == np.uint16:
+                a = a.view(np.int16)
+            return torch.from_numpy(a).to(dev)
+        self.tensors = {k: t(getattr(graph, k)) for k in
+                        ("row_ptr", "col", "ekind", "type", "warp", "cta", "work", "lat_extra", "cta_kernel",
+                         "node_off", "cta_off")}
+        n, m, C, W, G = graph.n_nodes, graph.n_edges, graph.n_ctas, graph.warps_per_cta, graph.n_graphs
+        nbytes = gts_graph_workspace_bytes(n, m, C, W, G)
+        if nbytes == 0:
+            raise GtsError(GTS_ERR_INVALID_ARG, "graph size out of range")
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        T = self.tensors
+        d = GraphDesc(n, m, C, W, G, T["node_off"].data_ptr(), T["cta_off"].data_ptr(), T["row_ptr"].data_ptr(),
+                      T["col"].data_ptr(), T["ekind"].data_ptr(), T["type"].data_ptr(), T["warp"].data_ptr(),
+                      T["cta"].data_ptr(), T["work"].data_ptr(), T["lat_extra"].data_ptr(),
+                      T["cta_kernel"].data_ptr(), self.workspace.data_ptr(), nbytes)
+        self.desc = d
+        self.handle = gts_graph_create(d, _stream_handle(stream))
+        self.row_nodes = gts_row_nodes(self.handle)
+        self.row_ctas = gts_row_ctas(self.handle)
+
+    def close(self):
+        if getattr(self, "handle", None):
+            gts_graph_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class DeviceParams:
+    """A [P][24] int32 parameter table resident on the GPU."""
+
+    def __init__(self, dgraph: DeviceGraph, params, stream=None):
+        import torch
+        self.dgraph = dgraph
+        p = np.ascontiguousarray(params, np.int32)
+        self.n_points = int(p.shape[0])
+        self.tensor = torch.from_numpy(p.reshape(-1)).to(dgraph.workspace.device)
+        self.handle = gts_params_upload(dgraph.handle, self.tensor.data_ptr(), self.n_points, _stream_handle(stream))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            gts_params_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+@dataclasses.dataclass
+class BatchOutput:
+    makespan: object
+    status: object
+    start: object = None
+    finish: object = None
+    digest: object = None
+    cta_sm: object = None
+
+
+def alloc_outputs(dgraph: DeviceGraph, n_points: int, flags: int):
+    import torch
+    dev = dgraph.workspace.device
+    out = BatchOutput(makespan=torch.empty(n_points, dtype=torch.int32, device=dev),
+                      status=torch.empty(n_points, dtype=torch.int32, device=dev))
+    if flags & GTS_FULL_TRACE:
+        out.start = torch.empty((n_points, dgraph.row_nodes), dtype=torch.int32, device=dev)
+        out.finish = torch.empty((n_points, dgraph.row_nodes), dtype=torch.int32, device=dev)
+    if flags & GTS_WANT_DIGEST:
+        out.digest = torch.empty(n_points, dtype=torch.int64, device=dev)
+    if flags & GTS_WANT_CTA_SM:
+        out.cta_sm = torch.empty((n_points, dgraph.row_ctas), dtype=torch.int32, device=dev)
+    return out
+
+
+def _ptr(t):
+    return 0 if t is None else t.data_ptr()
+
+
+def simulate(dgraph: DeviceGraph, dparams: DeviceParams, first_point=0, n_points=None,
+             flags=GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM, out: BatchOutput = None,
+             scratch=None, stream=None) -> BatchOutput:
+    """Enqueue one gts_simulate_batch on ``stream`` (default: torch's current)."""
+    import torch
+    if n_points is None:
+        n_points = dparams.n_points - first_point
+    if out is None:
+        out = alloc_outputs(dgraph, n_points, flags)
+    if scratch is None and not (flags & GTS_FULL_TRACE):
+        nb = gts_scratch_bytes(dgraph.handle, dparams.handle, flags)
+        scratch = torch.empty(max(nb, 16), dtype=torch.uint8, device=dgraph.workspace.device)
+    gts_simulate_batch(dgraph.handle, dparams.handle, first_point, n_points, flags, _ptr(out.start),
+                       _ptr(out.finish), _ptr(out.makespan), _ptr(out.status), _ptr(out.digest),
+                       _ptr(out.cta_sm), _ptr(scratch), 0 if scratch is None else scratch.numel(),
+                       _stream_handle(stream))
+    out.scratch = scratch
+    return out
