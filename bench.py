@@ -1,0 +1,323 @@
+"""Benchmark: batched tile-graph simulation throughput on GB300.
+
+One step = one gts_simulate_batch over every design point of the workload
+(full per-node start/finish trace), i.e. one pass of the whole hot path.
+Default workload: the warp-specialised persistent GEMM 8192^3 tile graph
+(1.58M nodes) x 4096 design points.  Prints ONE JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the CPU oracle on the host cores
+
+Under torchrun (N > 1) every rank simulates its own 4096 design points (drawn
+with a rank-specific seed) on its own GPU: no data-path collective; the
+per-rank times are reduced with a max at the end.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "simulated tile-graph nodes/sec"
+UNIT = "node-points/s"
+KERNEL_SRC = os.path.join(ROOT, "paper_2607_11262_gb300", "csrc", "gts.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_k_simulate.json")
+
+
+def node_points_of(graph, params):
+    """Simulated nodes summed over the design points (each point runs its graph)."""
+    if graph.n_graphs == 1:
+        return graph.n_nodes * int(params.shape[0])
+    sizes = np.diff(graph.node_off.astype(np.int64))
+    return int(sizes[params[:, 19]].sum())
+
+
+def algorithmic_bytes(graph, params, full_trace=True):
+    """Bytes the batch must move at minimum: the graph read once (node fields
+    1+2+4+4+4+2 B, row pointers, 5 B per edge), 96 B per parameter row, and per
+    point its trace (start + finish, 8 B per node), makespan and status."""
+    n, m = graph.n_nodes, graph.n_edges
+    graph_bytes = n * (1 + 2 + 4 + 4 + 4 + 2) + (n + 1) * 4 + m * 5
+    P = int(params.shape[0])
+    return graph_bytes + 96 * P + (8 * node_points_of(graph, params) if full_trace else 0) + 8 * P
+
+
+def source_hash():
+    return hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()[:16]
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clock and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"gts_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.dev}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(nm)
+        os.unlink(self.path)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def load_workload(name, rank, points):
+    from paper_2607_11262_gb300 import workloads as W
+    w = W.workload(name)
+    if rank > 0 and name != "stress":
+        # weak scaling: every rank gets its own design points of the same sweep
+        axes = {"gemm512": [W.AX_SMS, W.AX_HBM, (W.P_MMA_LAT, 16, 64)],
+                "wsgemm8192": [W.AX_SMS, W.AX_HBM, W.AX_TMA_LAT, W.AX_MMA_RATE]}.get(
+            name, [W.AX_SMS, W.AX_HBM, W.AX_TMA_LAT, W.AX_MMA_RATE, W.AX_ALU_RATE])
+        cps = int(w.params[0, W.P_CTAS_PER_SM])
+        w.params = W.sweep_params(W.SEED0 + 100 * rank + W.WORKLOADS.index(name) + 1, w.params.shape[0], axes, cps)
+    if points is not None:
+        w.params = w.params[:points]
+    return w
+
+
+def cpu_baseline(graph, params, seconds=15.0, procs=None):
+    """The oracle, as it stands, on the host cores over a bounded sample of the
+    workload's points (spawned worker processes, one point per process)."""
+    from oracle import run as oracle_run
+    procs = procs or (os.cpu_count() or 1)
+    t0 = time.time()
+    oracle_run.simulate(graph, params[0])       # one point to size the sample
+    t_one = time.time() - t0
+    k = int(max(1, min(params.shape[0], procs * max(1, round(seconds / max(t_one, 1e-3))))))
+    k = max(1, min(k, procs * 4))
+    pts = list(range(k))
+    t0 = time.time()
+    res = oracle_run.simulate_points(graph, params, pts, processes=min(procs, k))
+    wall = time.time() - t0
+    assert all(r.status == 0 for r in res.values())
+    nodes = node_points_of(graph, params[pts])
+    return {"value": nodes / wall, "unit": UNIT, "cores": min(procs, k), "kind": "oracle",
+            "sample": f"{k} of {params.shape[0]} design points, {min(procs, k)} processes, {wall:.1f} s wall"}
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    w = load_workload(args.workload, 0, args.points)
+    g = w.graph
+    vals, times = [], []
+    node_points = node_points_of(g, w.params)
+    for i in range(args.warmup + args.steps):
+        cb = cpu_baseline(g, w.params, seconds=args.ref_seconds)
+        if i >= args.warmup:
+            vals.append(cb["value"])
+            times.append(cb)
+    v = float(np.median(vals))
+    n = g.max_graph_nodes
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": node_points / v * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": w.name, "description": w.description, "nodes": n,
+                       "design_points": int(w.params.shape[0])},
+            "impl": "reference", "cpu_baseline": dict(times[-1], value=v),
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gts", choices=["gts", "reference"])
+    ap.add_argument("--workload", default="wsgemm8192")
+    ap.add_argument("--points", type=int, default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ref-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    from paper_2607_11262_gb300 import gts
+    gts.load()
+
+    w = load_workload(args.workload, rank, args.points)
+    g = w.graph
+    P = int(w.params.shape[0])
+    n = g.max_graph_nodes
+    node_points = node_points_of(g, w.params)
+    flags = gts.GTS_FULL_TRACE | gts.GTS_WANT_DIGEST
+    stream = torch.cuda.Stream()
+
+    with torch.cuda.stream(stream):
+        dg = gts.DeviceGraph(g, stream=stream)
+        dp = gts.DeviceParams(dg, w.params, stream=stream)
+        out = gts.alloc_outputs(dg, P, flags)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+
+    def barrier():
+        if ws > 1:
+            torch.distributed.barrier()
+
+    for _ in range(args.warmup):
+        gts.simulate(dg, dp, flags=flags, out=out, stream=stream)
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    clocks = Clocks(local)
+    clocks.start()
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        gts.simulate(dg, dp, flags=flags, out=out, stream=stream)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    ck = clocks.stop()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = float(sum(step_ms))
+    st = out.status.cpu().numpy()
+    assert np.all(st == 0), f"non-OK statuses: {np.unique(st)}"
+    if ws > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = node_points * ws / (ms_per_step / 1e3)
+
+    # ---- e2e: host buffers through the C ABI, copies inside the timed region
+    e2e = None
+    if rank == 0 or ws > 1:
+        e2e = measure_e2e(g, w.params, gts, stream)
+
+    if rank != 0:
+        if ws > 1:
+            torch.distributed.destroy_process_group()
+        return
+    alg = algorithmic_bytes(g, w.params)
+    kernel_s = ms_per_step / 1e3
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
+        os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
+    peak = float(peaks.get("hbm_gbs", 6800.0))
+    achieved = alg / kernel_s / 1e9
+    traffic = None
+    if os.path.exists(TRAFFIC_FILE):
+        tf = json.load(open(TRAFFIC_FILE))
+        if tf.get("source_sha256_16") == source_hash() and tf.get("workload") == w.name:
+            traffic = tf["bytes_per_node_point"] * node_points + tf.get("bytes_fixed", 0)
+    cb = None
+    if not args.no_cpu_baseline:
+        cb = cpu_baseline(g, w.params, seconds=args.ref_seconds)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int32", "data": "synthetic",
+        "config": {"workload": w.name, "description": w.description, "nodes": n, "edges": g.n_edges,
+                   "design_points_per_gpu": P, "full_trace": True,
+                   "l2": "inputs+outputs larger than L2 (trace rows alone exceed it)",
+                   "parallelism": f"design points sharded over {ws} GPU(s)"},
+        "design_points_per_s": P * ws / kernel_s,
+        "hbm_gbs_algorithmic": achieved,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_source": "measured" if peaks else "fallback",
+                     "frac_of_8tbps": achieved / 8000.0},
+        "cpu_baseline": cb, "e2e": e2e, "gpu_launches": args.steps, "clocks": ck,
+        "kernel_source": source_hash(),
+    }
+    print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def measure_e2e(graph, params, gts, stream, reps=2):
+    """Same metric through the public API from pinned host buffers: graph and
+    parameter upload (host->device), graph packing, the batch, and the
+    device->host read of the per-point makespans and statuses, every step."""
+    import torch
+    P = int(params.shape[0])
+    node_points = node_points_of(graph, params)
+    host = {k: torch.from_numpy(np.ascontiguousarray(getattr(graph, k)).view(
+        np.int32 if getattr(graph, k).dtype == np.uint32 else (np.int16 if getattr(graph, k).dtype == np.uint16
+                                                                else getattr(graph, k).dtype))).pin_memory()
+            for k in ("row_ptr", "col", "ekind", "type", "warp", "cta", "work", "lat_extra", "cta_kernel",
+                      "node_off", "cta_off")}
+    hp = torch.from_numpy(np.ascontiguousarray(params, np.int32).reshape(-1)).pin_memory()
+    h_mk = torch.empty(P, dtype=torch.int32).pin_memory()
+    h_st = torch.empty(P, dtype=torch.int32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in host.values()) + hp.numel() * 4
+    d2h = P * 8
+    flags = gts.GTS_FULL_TRACE
+    times = []
+    dev = torch.device("cuda")
+    for _ in range(reps):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            dt = {k: v.to(dev, non_blocking=True) for k, v in host.items()}
+            dpar = hp.to(dev, non_blocking=True)
+            dg = gts.DeviceGraph.from_device_tensors(graph, dt, stream=stream)
+            dpp = gts.DeviceParams.from_device_tensor(dg, dpar, P, stream=stream)
+            out = gts.alloc_outputs(dg, P, flags)
+            gts.simulate(dg, dpp, flags=flags, out=out, stream=stream)
+            h_mk.copy_(out.makespan, non_blocking=True)
+            h_st.copy_(out.status, non_blocking=True)
+        stream.synchronize()
+        times.append(time.perf_counter() - t0)
+        del out, dpp, dg, dt, dpar
+    t = min(times)
+    return {"value": node_points / t, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "seconds_per_step": t}
+
+
+if __name__ == "__main__":
+    main()

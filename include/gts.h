@@ -124,7 +124,8 @@ typedef struct gts_results gts_results;
  *  - type < 7, warp < warps_per_cta, cta inside the node's graph;
  *  - cta_kernel is non-decreasing within each graph.
  * The program order of each (cta, warp) stream is ascending id.
- * Limits: n_nodes < 2^31, n_ctas < 2^24, warps_per_cta <= 128.
+ * Limits: n_nodes < 2^31, n_ctas < 2^24, warps_per_cta <= 128, in-degree
+ * < 2^24 (GTS_ERR_UNSUPPORTED beyond).
  */
 typedef struct {
   uint32_t n_nodes, n_edges, n_ctas, warps_per_cta, n_graphs;
@@ -172,10 +173,12 @@ gts_status gts_params_destroy(gts_params *params);
 uint32_t gts_row_nodes(const gts_graph *graph);
 uint32_t gts_row_ctas(const gts_graph *graph);
 
-/* Device scratch gts_simulate_batch wants for `flags`: without GTS_FULL_TRACE
- * the per-warp start/finish rows live in scratch; with it, none is needed.
- * Returns the size that lets every resident warp work; a smaller non-zero
- * scratch runs fewer design points at a time. */
+/* Device scratch gts_simulate_batch wants: one row of dependency counters per
+ * concurrently simulated design point (8 bytes per node of the largest graph,
+ * rounded up to 16 bytes).  Returns the size that lets every resident warp
+ * work; a smaller scratch (at least one row) runs fewer points at a time.
+ * The kernel clears each row itself; its contents between calls are
+ * irrelevant.  Calls sharing one scratch must not overlap on the GPU. */
 size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint32_t flags);
 
 /*
@@ -188,8 +191,10 @@ size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint3
  * Start/finish/digest/cta_sm of a point whose status is not GTS_OK are
  * unspecified.  The digest is sum over v of splitmix64-finalise(
  * (v << 32 | (uint32)start) ^ ((uint64)(uint32)finish * 0x9E3779B97F4A7C15)) mod 2^64.
- * Enqueues on `stream` and returns; *out (may be NULL) remembers the arrays
- * for gts_read_results.  Errors: INVALID_ARG, NOMEM (scratch too small), CUDA.
+ * d_scratch (16-byte aligned, scratch_bytes long) is required; see
+ * gts_scratch_bytes.  Enqueues on `stream` and returns; *out (may be NULL)
+ * remembers the arrays for gts_read_results.  Errors: INVALID_ARG, NOMEM
+ * (scratch smaller than one row), CUDA.
  */
 gts_status gts_simulate_batch(gts_graph *graph, gts_params *params,
                               uint32_t first_point, uint32_t n_points, uint32_t flags,

@@ -1,35 +1,51 @@
 // gts.cu -- libgts: batched graph-driven tile-graph simulation on sm_103a.
 //
 // One warp simulates one design point (one hardware parameter row) of the
-// graph-driven simulation backend (Section 5): the warp keeps the event
-// frontier -- the head node of every logical warp stream of every resident
-// CTA -- plus the per-SM unit servers, the global HBM servers and the CTA
-// slots in shared memory, and advances the schedule with warp ballot / shuffle
-// / min-reduction primitives.  The tile graph is shared read-only by all
-// points; each point's start/finish rows live in global memory (the output
-// trace, or caller scratch).
+// graph-driven simulation backend (Section 5).  The warp keeps in shared
+// memory the event frontier -- the head node of every logical warp stream of
+// every resident CTA -- with a cached issue key per head, the per-SM unit
+// servers, the global HBM servers, the CTA slots, and one summary per
+// simulated SM; it advances the schedule with warp min-reductions.  The tile
+// graph is shared read-only by all points.  Per point, a global scratch row
+// holds the dependency counters of nodes that are not warp heads yet.
 //
 // Semantics are those stated in include/gts.h.  Design notes:
-//  * Issue selection (Section 5.3, lowest-id reading): every frontier slot
-//    caches key = max(rdy, earliest free server of its per-SM class), or INF
-//    while a predecessor is unissued; a head is issuable at t when key <= t
-//    and, for LOAD/STORE, some HBM server is free at t.  The warp takes the
-//    minimum node id over issuable heads (one __reduce_min_sync).
-//  * Dependency release (Section 5.1): an issued node pushes its release time
-//    (issue cycle for ISSUE edges, finish for DATA edges) only into
-//    successors that are currently warp heads; a node that becomes a head
-//    pulls the state of its already-issued predecessors from the point's
-//    start/finish rows (start = -1 marks "not issued").  Every predecessor is
-//    thus counted exactly once.
-//  * Time advance: the next cycle is the minimum over heads of their key
-//    (raised to the HBM availability for LOAD/STORE) and over finished CTAs of
-//    their retirement cycle; no cycle in between can issue or launch.
+//  * Issue keys (Section 5.3, lowest-id reading).  A head's key is the
+//    earliest cycle >= now at which its predecessors are released and its
+//    per-SM unit has a free server (INF while a predecessor is unissued); for
+//    LOAD/STORE the effective cycle is max(key, H), H the earliest free HBM
+//    server.  Every unissued head keeps effective cycle >= t (keys are clamped
+//    to the cycle they are computed at; a head that could issue at t but did
+//    not has had its key recomputed when its unit or H changed), so the next
+//    event is the lexicographic minimum of (effective cycle, node id) over
+//    all heads: if that cycle is t, the node is the lowest-id issuable head;
+//    otherwise it is the next event cycle.  Lane l owns simulated SMs
+//    l, l+32, ...; each SM keeps the (cycle, id) minimum of its non-HBM heads
+//    and of its HBM heads in shared memory, each lane the minimum over its SMs
+//    in registers, and the warp takes the minimum over lanes with two
+//    __reduce_min_sync.  After an issue only the issuing SM's owner lane
+//    recomputes (all lanes when H moved).
+//  * The issue itself runs in every lane on broadcast values (no divergence);
+//    only global atomics and scratch-counter reads are lane 0's.
+//  * Dependency release (Section 5.1).  An issued node releases each
+//    successor at its issue cycle (ISSUE edge) or finish (DATA edge): into the
+//    frontier if the successor is a warp head, else into the successor's
+//    scratch counters (count of released predecessors, max release cycle)
+//    with fire-and-forget global atomics.  A node that becomes a head reads
+//    its counters once; everything after that reaches it in shared memory.
+//    Lane 0 performs every release and every counter read of a point, so
+//    program order orders them; CTA launches, whose heads are read by other
+//    lanes, fence first.
+//  * Occupancy ceil(work / rate) uses exact division by invariant integers
+//    (Lemire, Kaser, Kurz 2019: floor(n/d) = floor(ceil(2^64/d) * n / 2^64)
+//    for 32-bit n and d), with the per-point constants computed once.
 //  * Server identity is unobservable, so "take any free server" takes the
 //    first free one.
 //  * Every loop is bounded: the per-point step count is capped by
 //    8*n + 4*C + 64 (each step launches a CTA, issues a node or moves to a
-//    distinct finish / server-free cycle, of which there are at most 3n);
-//    reaching it writes GTS_ERR_STEP_LIMIT.  No kernel waits on another.
+//    distinct finish / server-free / retirement cycle, of which there are at
+//    most 3n); reaching it writes GTS_ERR_STEP_LIMIT.  No warp waits on
+//    another warp.
 #include "gts.h"
 
 #include <cuda_runtime.h>
@@ -51,9 +67,16 @@ constexpr uint32_t FULL = 0xFFFFFFFFu;
 constexpr int MAX_WPB = 4;                  // warps (design points) per block
 constexpr uint32_t MAX_SMEM_BYTES = 227u * 1024u;
 constexpr uint32_t MAX_W = 128;
+constexpr uint32_t MAX_INDEG = (1u << 24) - 1;
+constexpr uint32_t DEG_BIG = 31;            // successor count field: 31 = read it from the graph
 
 // per-SM resource classes (Section 5.2)
 enum : uint32_t { RC_TENSOR = 0, RC_TMA = 1, RC_LSU = 2, RC_ALU = 3, RC_BAR = 4, RC_N = 5, RC_NONE = 7 };
+// rates with a division constant
+enum : uint32_t { RT_HBM = 0, RT_TMA = 1, RT_SMEM = 2, RT_MMA = 3, RT_ALU = 4 };
+static_assert(GTS_P_TMA_BPC == GTS_P_HBM_BPC + 2 && GTS_P_SMEM_BPC == GTS_P_HBM_BPC + 4 &&
+                  GTS_P_MMA_FMA_PC == GTS_P_HBM_BPC + 6 && GTS_P_ALU_OPS_PC == GTS_P_HBM_BPC + 8,
+              "rate k of the division-constant table sits at parameter index GTS_P_HBM_BPC + 2k");
 
 thread_local std::string g_err;
 
@@ -68,10 +91,9 @@ gts_status cuda_fail(cudaError_t e, const char *what) {
 
 // ----------------------------------------------------------------- device graph
 struct DevGraph {
-  const uint4 *rec;            // [n] x=work y=lat_extra z=next node of the stream w=type|warp<<4
-  const uint4 *rng;            // [n] x,y = predecessor list range; z,w = successor list range
+  const uint4 *rec;            // [n] x=work y=lat_extra z=next node of the stream w=type | indegree<<4
+  const uint4 *rng;            // [n] z,w = successor list range (x, y unused)
   const uint2 *succ;           // [m] x=successor id, y=kind | warp<<1 | cta<<8
-  const uint32_t *pred;        // [m] predecessor id | kind<<31
   const uint32_t *stream_first;// [C*W] first node of stream (c, w) or NONE
   const uint32_t *cta_cnt;     // [C] nodes per CTA
   const uint32_t *cta_kernel;  // [C]
@@ -81,15 +103,19 @@ struct DevGraph {
 };
 
 // ----------------------------------------------------------------- per-point layout
-// Shared-memory words of one design point.  Frontier slot s = (cta slot) * W
-// + warp; CTA slot j lives on SM j / ctas_per_sm (SM-major, so the lowest free
+// Shared-memory words of one design point.  Frontier slot i = (CTA slot) * W +
+// warp; CTA slot j lives on SM j / ctas_per_sm (SM-major, so the lowest free
 // slot is on the lowest SM with room).  Only min(num_sms*cps, C) CTA slots can
 // ever be occupied (a launch always takes the lowest free slot).
+constexpr uint32_t O_CAP = GTS_NPARAM;       // 5 words: servers per class
+constexpr uint32_t O_OFF = GTS_NPARAM + 5;   // 5 words: class offset inside an SM's servers
+constexpr uint32_t O_MAG = GTS_NPARAM + 10;  // 5 x 2 words: division constants of the rates
+constexpr uint32_t O_DYN = GTS_NPARAM + 20;  // first per-point array (even: 8-byte aligned)
+constexpr uint32_t SM_WORDS = 6;             // per SM: lo key, lo id, lo slot, hbm key, hbm id, hbm slot
+
 struct Layout {
-  uint32_t S, Scta, NS, SC, cap_hbm;
-  uint32_t cap[RC_N], off[RC_N];
-  uint32_t o_prm, o_hid, o_key, o_rdy, o_np, o_L, o_occ, o_hocc, o_next, o_sb, o_se, o_meta;
-  uint32_t o_cid, o_crem, o_cend, o_ckern, o_sv, o_hs, words;
+  uint32_t S, Scta, NS, SC, cap_hbm, per;
+  uint32_t o_hid, o_key, o_rdy, o_meta, o_nxt, o_sb, o_sm, o_cid, o_crem, o_cend, o_ckern, o_sv, o_hs, words;
 };
 
 __host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
@@ -109,7 +135,8 @@ __host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
 }
 
 // Fills `L` for a valid row on a graph with CG CTAs; false if the point needs
-// more than one warp's shared-memory budget.
+// more than one warp's shared-memory budget.  Servers per class are limited
+// to 32 (one lane each).
 __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint32_t W, Layout &L) {
   const uint64_t cps = (uint64_t)p[GTS_P_CTAS_PER_SM];
   uint64_t slots = (uint64_t)p[GTS_P_NUM_SMS] * cps;
@@ -117,30 +144,25 @@ __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint3
   L.Scta = (uint32_t)slots;
   L.S = L.Scta * W;
   L.NS = (uint32_t)((slots + cps - 1) / cps);
+  if (cps * W > 0xFFFFull) return false;
+  L.per = (uint32_t)(cps * W);
   uint64_t sc = 0;
   for (int r = 0; r < (int)RC_N; r++) {
     const uint64_t c = (uint64_t)p[GTS_P_CAP_TENSOR + r];
-    if (c > 65536) return false;
-    L.cap[r] = (uint32_t)c;
-    L.off[r] = (uint32_t)sc;
+    if (c > 32) return false;
     sc += c;
   }
   L.SC = (uint32_t)sc;
-  if ((uint64_t)p[GTS_P_CAP_HBM] > 65536) return false;
+  if ((uint64_t)p[GTS_P_CAP_HBM] > 32) return false;
   L.cap_hbm = (uint32_t)p[GTS_P_CAP_HBM];
-  uint64_t w = 0;
-  L.o_prm = (uint32_t)w; w += GTS_NPARAM;
+  uint64_t w = O_DYN;
   L.o_hid = (uint32_t)w; w += L.S;
   L.o_key = (uint32_t)w; w += L.S;
   L.o_rdy = (uint32_t)w; w += L.S;
-  L.o_np = (uint32_t)w; w += L.S;
-  L.o_L = (uint32_t)w; w += L.S;
-  L.o_occ = (uint32_t)w; w += L.S;
-  L.o_hocc = (uint32_t)w; w += L.S;
-  L.o_next = (uint32_t)w; w += L.S;
-  L.o_sb = (uint32_t)w; w += L.S;
-  L.o_se = (uint32_t)w; w += L.S;
   L.o_meta = (uint32_t)w; w += L.S;
+  L.o_nxt = (uint32_t)w; w += L.S;
+  L.o_sb = (uint32_t)w; w += L.S;
+  L.o_sm = (uint32_t)w; w += (uint64_t)L.NS * SM_WORDS;
   L.o_cid = (uint32_t)w; w += L.Scta;
   L.o_crem = (uint32_t)w; w += L.Scta;
   L.o_cend = (uint32_t)w; w += L.Scta;
@@ -154,7 +176,15 @@ __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint3
 }
 
 // ----------------------------------------------------------------- device helpers
-__device__ __forceinline__ uint32_t cdiv(uint32_t a, uint32_t b) { return a / b + (a % b != 0u); }
+// ceil(2^64 / d) for d >= 2 (0 encodes d == 1).
+__device__ __forceinline__ uint64_t div_const(uint32_t d) { return d <= 1u ? 0ull : ~0ull / d + 1ull; }
+
+// ceil(n / d) given M = div_const(d).
+__device__ __forceinline__ uint32_t cdiv_c(uint32_t n, uint32_t d, uint64_t M) {
+  if (M == 0ull) return n;
+  const uint32_t q = (uint32_t)__umul64hi(M, (uint64_t)n);
+  return q + (q * d != n ? 1u : 0u);
+}
 
 __device__ __forceinline__ uint64_t mix64(uint64_t z) {  // splitmix64 finaliser (Steele, Lea, Flood 2014)
   z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
@@ -162,157 +192,171 @@ __device__ __forceinline__ uint64_t mix64(uint64_t z) {  // splitmix64 finaliser
   return z ^ (z >> 31);
 }
 
-struct Point {
-  uint32_t *sp;      // this warp's shared-memory words
-  Layout L;
-  uint32_t W, cps, n0, c0, c1;
-  int32_t *st, *fi;  // point rows (graph-local index)
-};
-
-// Per-node unit, occupancy and latency (Section 5.2 throughput model).
-__device__ __forceinline__ void node_cost(const Point &P, uint32_t type, uint32_t work, uint32_t lx, uint32_t &cls,
-                                          uint32_t &occ, uint32_t &hocc, uint32_t &lat, bool &hbm) {
-  const int32_t *prm = reinterpret_cast<const int32_t *>(P.sp + P.L.o_prm);
-  uint32_t base = 0;
-  cls = RC_NONE;
-  occ = 0;
-  hocc = 0;
-  hbm = false;
-  switch (type) {
-    case GTS_LOAD:
-      cls = RC_TMA; occ = cdiv(work, (uint32_t)prm[GTS_P_TMA_BPC]);
-      hbm = true; hocc = cdiv(work, (uint32_t)prm[GTS_P_HBM_BPC]);
-      base = (uint32_t)prm[GTS_P_TMA_LAT] + (uint32_t)prm[GTS_P_DRAM_LAT];
-      break;
-    case GTS_SMEM:
-      cls = RC_LSU; occ = cdiv(work, (uint32_t)prm[GTS_P_SMEM_BPC]); base = (uint32_t)prm[GTS_P_SMEM_LAT];
-      break;
-    case GTS_MMA:
-      cls = RC_TENSOR; occ = cdiv(work, (uint32_t)prm[GTS_P_MMA_FMA_PC]); base = (uint32_t)prm[GTS_P_MMA_LAT];
-      break;
-    case GTS_EW:
-      cls = RC_ALU; occ = cdiv(work, (uint32_t)prm[GTS_P_ALU_OPS_PC]); base = (uint32_t)prm[GTS_P_ALU_LAT];
-      break;
-    case GTS_STORE:
-      cls = RC_TMA; occ = cdiv(work, (uint32_t)prm[GTS_P_TMA_BPC]);
-      hbm = true; hocc = cdiv(work, (uint32_t)prm[GTS_P_HBM_BPC]);
-      base = (uint32_t)prm[GTS_P_TMA_LAT];
-      break;
-    case GTS_BAR:
-      cls = RC_BAR; occ = 1; base = (uint32_t)prm[GTS_P_BAR_LAT];
-      break;
-    default:
-      break;
-  }
-  const uint64_t L = (uint64_t)base + lx + (occ > hocc ? occ : hocc);
-  lat = L > 0x80000000ull ? 0x80000000u : (uint32_t)L;  // any value >= 2^31 overflows at issue
+__device__ __forceinline__ uint2 ld_counters(const uint2 *p) {  // strong load of a scratch counter pair
+  uint2 r;
+  asm volatile("ld.relaxed.gpu.global.v2.u32 {%0, %1}, [%2];" : "=r"(r.x), "=r"(r.y) : "l"(p) : "memory");
+  return r;
 }
 
-// Earliest cycle slot i's head could issue, ignoring HBM; INF if blocked.
-__device__ __forceinline__ uint32_t slot_key(const Point &P, uint32_t i) {
+struct Pt {
+  uint32_t *sp;  // this warp's shared-memory words
+  Layout L;
+  uint32_t W, cps, n0, c0, c1;
+  int32_t *st, *fi;  // trace rows (graph-local index) or null
+  uint2 *scr;        // scratch counters (graph-local index)
+};
+
+// Per-SM class and HBM use of a node type (Section 4.1 operation descriptor).
+__device__ __forceinline__ uint32_t type_class(uint32_t type) {
+  switch (type) {
+    case GTS_LOAD: case GTS_STORE: return RC_TMA;
+    case GTS_SMEM: return RC_LSU;
+    case GTS_MMA: return RC_TENSOR;
+    case GTS_EW: return RC_ALU;
+    case GTS_BAR: return RC_BAR;
+    default: return RC_NONE;
+  }
+}
+__device__ __forceinline__ bool type_hbm(uint32_t type) { return type == GTS_LOAD || type == GTS_STORE; }
+
+__device__ __forceinline__ uint32_t rate_occ(const uint32_t *sp, uint32_t work, uint32_t rt, int pidx) {
+  const uint64_t M = *reinterpret_cast<const uint64_t *>(sp + O_MAG + 2 * rt);
+  return cdiv_c(work, sp[pidx], M);
+}
+
+// Occupancies and latency of a node (Section 5.2 throughput model).
+__device__ __forceinline__ void node_cost(const uint32_t *sp, uint32_t type, uint32_t work, uint32_t lx,
+                                          uint32_t &occ, uint32_t &hocc, uint64_t &lat) {
+  uint32_t base = 0;
+  occ = 0;
+  hocc = 0;
+  switch (type) {
+    case GTS_LOAD:
+      occ = rate_occ(sp, work, RT_TMA, GTS_P_TMA_BPC);
+      hocc = rate_occ(sp, work, RT_HBM, GTS_P_HBM_BPC);
+      base = sp[GTS_P_TMA_LAT] + sp[GTS_P_DRAM_LAT];
+      break;
+    case GTS_SMEM: occ = rate_occ(sp, work, RT_SMEM, GTS_P_SMEM_BPC); base = sp[GTS_P_SMEM_LAT]; break;
+    case GTS_MMA: occ = rate_occ(sp, work, RT_MMA, GTS_P_MMA_FMA_PC); base = sp[GTS_P_MMA_LAT]; break;
+    case GTS_EW: occ = rate_occ(sp, work, RT_ALU, GTS_P_ALU_OPS_PC); base = sp[GTS_P_ALU_LAT]; break;
+    case GTS_STORE:
+      occ = rate_occ(sp, work, RT_TMA, GTS_P_TMA_BPC);
+      hocc = rate_occ(sp, work, RT_HBM, GTS_P_HBM_BPC);
+      base = sp[GTS_P_TMA_LAT];
+      break;
+    case GTS_BAR: occ = 1; base = sp[GTS_P_BAR_LAT]; break;
+    default: break;
+  }
+  lat = (uint64_t)base + lx + (occ > hocc ? occ : hocc);
+}
+
+// Key of slot i computed at cycle t (>= t; INF if it cannot issue yet).
+__device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t) {
   const uint32_t *sp = P.sp;
   const uint32_t h = sp[P.L.o_hid + i];
-  if (h == NONE || sp[P.L.o_np + i] != 0u) return INF;
-  uint32_t k = sp[P.L.o_rdy + i];
-  const uint32_t cls = sp[P.L.o_meta + i] & 7u;
+  const uint32_t meta = sp[P.L.o_meta + i];
+  if (h == NONE || (meta >> 8) != 0u) return INF;
+  uint32_t k = max(sp[P.L.o_rdy + i], t);
+  const uint32_t cls = meta & 7u;
   if (cls != RC_NONE) {
-    const uint32_t sm = (i / P.W) / P.cps;
-    const uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + P.L.off[cls];
+    const uint32_t sm = i / P.L.per;
+    const uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + sp[O_OFF + cls];
+    const uint32_t cap = sp[O_CAP + cls];
     uint32_t a = sv[0];
-    for (uint32_t q = 1; q < P.L.cap[cls]; q++) a = min(a, sv[q]);
+    for (uint32_t q = 1; q < cap; q++) a = min(a, sv[q]);
     k = max(k, a);
   }
   return k;
 }
 
-// Slot i takes node v as its head (v == NONE: stream exhausted).  The caller's
-// lane alone does the work (used for CTA launches: one lane per stream).
-__device__ void load_head_lane(const DevGraph &g, const Point &P, uint32_t i, uint32_t v) {
+__device__ __forceinline__ bool lex_less(uint32_t k1, uint32_t id1, uint32_t k2, uint32_t id2) {
+  return k1 < k2 || (k1 == k2 && id1 < id2);
+}
+
+// Recomputes the summary of SM s from its slots' keys (one lane).
+__device__ void sm_summary(const Pt &P, uint32_t s, uint32_t H) {
+  uint32_t *sp = P.sp;
+  uint32_t lk = INF, lid = NONE, lsl = 0, hk = INF, hid = NONE, hsl = 0;
+  const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
+  for (uint32_t i = i0; i < i1; i++) {
+    const uint32_t k = sp[P.L.o_key + i];
+    const uint32_t h = sp[P.L.o_hid + i];
+    if (k == INF) continue;
+    const uint32_t id = h & ID_MASK;
+    if (h & HBM_BIT) {
+      const uint32_t e = max(k, H);
+      if (lex_less(e, id, hk, hid)) { hk = e; hid = id; hsl = i; }
+    } else if (lex_less(k, id, lk, lid)) {
+      lk = k; lid = id; lsl = i;
+    }
+  }
+  uint32_t *o = sp + P.L.o_sm + s * SM_WORDS;
+  o[0] = lk; o[1] = lid; o[2] = lsl; o[3] = hk; o[4] = hid; o[5] = hsl;
+}
+
+struct Summary {
+  uint32_t k, id, sl;
+};
+
+// The lane's minimum over the SMs it owns.
+__device__ __forceinline__ Summary lane_summary(const Pt &P, int lane) {
+  Summary b{INF, NONE, 0};
+  for (uint32_t s = lane; s < P.L.NS; s += 32) {
+    const uint32_t *o = P.sp + P.L.o_sm + s * SM_WORDS;
+    if (lex_less(o[0], o[1], b.k, b.id)) b = Summary{o[0], o[1], o[2]};
+    if (lex_less(o[3], o[4], b.k, b.id)) b = Summary{o[3], o[4], o[5]};
+  }
+  return b;
+}
+
+// Slot i takes node v as its head (v == NONE: stream exhausted); adj_cnt /
+// adj_rdy are releases the caller applied directly.  Every lane writes the
+// same values.
+__device__ __forceinline__ void set_head(const Pt &P, uint32_t i, uint32_t v, uint4 r, uint4 q, uint2 c,
+                                         uint32_t adj_cnt, uint32_t adj_rdy) {
   uint32_t *sp = P.sp;
   if (v == NONE) {
     sp[P.L.o_hid + i] = NONE;
     sp[P.L.o_key + i] = INF;
+    sp[P.L.o_meta + i] = RC_NONE;
     return;
   }
-  const uint4 r = g.rec[v];
-  const uint4 q = g.rng[v];
-  uint32_t cnt = 0;
-  int32_t rdy = 0;
-  for (uint32_t e = q.x; e < q.y; e++) {
-    const uint32_t pe = g.pred[e];
-    const uint32_t u = (pe & ID_MASK) - P.n0;
-    const int32_t s = P.st[u];
-    if (s < 0) cnt++;
-    else rdy = max(rdy, (pe >> 31) ? s : P.fi[u]);
-  }
-  uint32_t cls, occ, hocc, lat;
-  bool hbm;
-  node_cost(P, r.w & 15u, r.x, r.y, cls, occ, hocc, lat, hbm);
-  sp[P.L.o_hid + i] = v | (hbm ? HBM_BIT : 0u);
-  sp[P.L.o_np + i] = cnt;
-  sp[P.L.o_rdy + i] = (uint32_t)rdy;
-  sp[P.L.o_L + i] = lat;
-  sp[P.L.o_occ + i] = occ;
-  sp[P.L.o_hocc + i] = hocc;
-  sp[P.L.o_next + i] = r.z;
+  const uint32_t type = r.w & 15u;
+  const uint32_t pend = (r.w >> 4) - c.x - adj_cnt;
+  const uint32_t deg = min(q.w - q.z, DEG_BIG);
+  sp[P.L.o_hid + i] = v | (type_hbm(type) ? HBM_BIT : 0u);
+  sp[P.L.o_rdy + i] = max(c.y, adj_rdy);
+  sp[P.L.o_meta + i] = type_class(type) | (deg << 3) | (pend << 8);
+  sp[P.L.o_nxt + i] = r.z;
   sp[P.L.o_sb + i] = q.z;
-  sp[P.L.o_se + i] = q.w;
-  sp[P.L.o_meta + i] = cls;
 }
 
-// Same, with the whole warp pulling the predecessors (one per lane).
-__device__ void load_head_warp(const DevGraph &g, const Point &P, uint32_t i, uint32_t v, int lane) {
-  uint32_t *sp = P.sp;
-  if (v == NONE) {
-    if (lane == 0) {
-      sp[P.L.o_hid + i] = NONE;
-      sp[P.L.o_key + i] = INF;
-    }
-    return;
-  }
-  const uint4 r = g.rec[v];
-  const uint4 q = g.rng[v];
-  uint32_t cnt = 0;
-  int32_t rdy = 0;
-  for (uint32_t e = q.x + lane; e < q.y; e += 32) {
-    const uint32_t pe = g.pred[e];
-    const uint32_t u = (pe & ID_MASK) - P.n0;
-    const int32_t s = P.st[u];
-    if (s < 0) cnt++;
-    else rdy = max(rdy, (pe >> 31) ? s : P.fi[u]);
-  }
-  cnt = __reduce_add_sync(FULL, cnt);
-  rdy = __reduce_max_sync(FULL, rdy);
-  if (lane == 0) {
-    uint32_t cls, occ, hocc, lat;
-    bool hbm;
-    node_cost(P, r.w & 15u, r.x, r.y, cls, occ, hocc, lat, hbm);
-    sp[P.L.o_hid + i] = v | (hbm ? HBM_BIT : 0u);
-    sp[P.L.o_np + i] = cnt;
-    sp[P.L.o_rdy + i] = (uint32_t)rdy;
-    sp[P.L.o_L + i] = lat;
-    sp[P.L.o_occ + i] = occ;
-    sp[P.L.o_hocc + i] = hocc;
-    sp[P.L.o_next + i] = r.z;
-    sp[P.L.o_sb + i] = q.z;
-    sp[P.L.o_se + i] = q.w;
-    sp[P.L.o_meta + i] = cls;
-  }
-}
+struct Clock {
+  uint32_t t;          // current cycle
+  uint32_t H;          // earliest free HBM server
+  uint32_t next_ret;   // earliest retirement cycle among finished, still resident CTAs
+  uint32_t next_cta;   // next CTA to launch (global id)
+  uint64_t steps, limit;
+};
 
 // Retire finished CTAs and launch as many CTAs as fit at cycle t (Section 5.1
-// TB scheduler; kernel-boundary gate).  Returns false on step-limit.
-__device__ bool launch_ctas(const DevGraph &g, Point &P, int32_t t, uint32_t &next_cta, uint64_t &steps,
-                            uint64_t step_limit, int32_t *cta_sm_row, int lane) {
+// TB scheduler; kernel-boundary gate).  Returns false on step-limit.  The
+// caller's lane summary `b` is refreshed when the lane owns a touched SM.
+__device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_row, int lane, Summary &b) {
   uint32_t *sp = P.sp;
+  const uint32_t t = C.t;
   for (;;) {
+    uint32_t nr = INF;
     for (uint32_t j = lane; j < P.L.Scta; j += 32) {
-      if (sp[P.L.o_cid + j] != NONE && sp[P.L.o_crem + j] == 0u && (int32_t)sp[P.L.o_cend + j] <= t)
-        sp[P.L.o_cid + j] = NONE;
+      if (sp[P.L.o_cid + j] != NONE && sp[P.L.o_crem + j] == 0u) {
+        if (sp[P.L.o_cend + j] <= t) sp[P.L.o_cid + j] = NONE;
+        else nr = min(nr, sp[P.L.o_cend + j]);
+      }
     }
+    C.next_ret = __reduce_min_sync(FULL, nr);
     __syncwarp();
-    if (next_cta >= P.c1) return true;
-    const uint32_t kc = g.cta_kernel[next_cta];
+    if (C.next_cta >= P.c1) return true;
+    const uint32_t kc = g.cta_kernel[C.next_cta];
     bool blocked = false;
     uint32_t freeslot = NONE;
     for (uint32_t j = lane; j < P.L.Scta; j += 32) {
@@ -325,37 +369,57 @@ __device__ bool launch_ctas(const DevGraph &g, Point &P, int32_t t, uint32_t &ne
     if (__any_sync(FULL, blocked)) return true;
     freeslot = __reduce_min_sync(FULL, freeslot);
     if (freeslot == NONE) return true;
-    if (++steps > step_limit) return false;
+    if (++C.steps > C.limit) return false;
+    const uint32_t c = C.next_cta;
+    const uint32_t cnt = g.cta_cnt[c];
     if (lane == 0) {
-      sp[P.L.o_cid + freeslot] = next_cta;
-      sp[P.L.o_crem + freeslot] = g.cta_cnt[next_cta];
+      sp[P.L.o_cid + freeslot] = c;
+      sp[P.L.o_crem + freeslot] = cnt;
       sp[P.L.o_cend + freeslot] = 0u;
       sp[P.L.o_ckern + freeslot] = kc;
-      if (cta_sm_row) cta_sm_row[next_cta - P.c0] = (int32_t)(freeslot / P.cps);
-    }
-    for (uint32_t w = lane; w < P.W; w += 32) {
-      const uint32_t i = freeslot * P.W + w;
-      load_head_lane(g, P, i, g.stream_first[(size_t)next_cta * P.W + w]);
-      sp[P.L.o_key + i] = slot_key(P, i);
+      if (cta_sm_row) cta_sm_row[c - P.c0] = (int32_t)(freeslot / P.cps);
+      __threadfence();  // lane 0's earlier counter releases before the heads are read below
     }
     __syncwarp();
-    next_cta++;
+    __threadfence();
+    for (uint32_t w = lane; w < P.W; w += 32) {
+      const uint32_t i = freeslot * P.W + w;
+      const uint32_t v = g.stream_first[(size_t)c * P.W + w];
+      uint4 r = make_uint4(0, 0, 0, 0), q = r;
+      uint2 cc = make_uint2(0, 0);
+      if (v != NONE) {
+        r = g.rec[v];
+        q = g.rng[v];
+        cc = ld_counters(P.scr + (v - P.n0));
+      }
+      set_head(P, i, v, r, q, cc, 0u, 0u);
+      sp[P.L.o_key + i] = slot_key(P, i, t);
+    }
+    __syncwarp();
+    const uint32_t s = freeslot / P.cps;
+    if ((uint32_t)lane == (s & 31u)) {
+      sm_summary(P, s, C.H);
+      b = lane_summary(P, lane);
+    }
+    __syncwarp();
+    C.next_cta++;
   }
 }
 
 __global__ void __launch_bounds__(MAX_WPB * 32)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
-           int32_t *d_cta_sm, int32_t *scratch, uint32_t n_warps, uint32_t budget_words) {
+           int32_t *d_cta_sm, uint2 *scratch, uint32_t n_warps, uint32_t budget_words) {
   extern __shared__ __align__(16) uint32_t smem[];
   const int lane = threadIdx.x & 31;
   const uint32_t wib = threadIdx.x >> 5;
   const uint32_t gw = blockIdx.x * (blockDim.x >> 5) + wib;
   if (gw >= n_warps) return;
-  Point P;
+  Pt P;
   P.sp = smem + wib * budget_words;
   P.W = g.W;
   uint32_t *sp = P.sp;
+  const bool want_digest = d_digest != nullptr;
 
   for (uint32_t q = gw; q < n_points; q += n_warps) {
     const uint32_t p = first_point + q;
@@ -366,10 +430,10 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     int status = check_row(prm, g.G);
     const uint32_t gi = status == GTS_OK ? (uint32_t)prm[GTS_P_GRAPH_INDEX] : 0u;
     P.n0 = g.node_off[gi];
-    const uint32_t n1 = g.node_off[gi + 1];
+    const uint32_t nG = g.node_off[gi + 1] - P.n0;
     P.c0 = g.cta_off[gi];
     P.c1 = g.cta_off[gi + 1];
-    const uint32_t nG = n1 - P.n0, CG = P.c1 - P.c0;
+    const uint32_t CG = P.c1 - P.c0;
     if (status == GTS_OK) {
       if (!make_layout(prm, CG, P.W, P.L) || P.L.words > budget_words) status = GTS_ERR_UNSUPPORTED;
     }
@@ -377,182 +441,215 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       if (lane == 0) {
         d_status[q] = status;
         d_makespan[q] = 0;
-        if (d_digest) d_digest[q] = 0;
+        if (want_digest) d_digest[q] = 0;
       }
       __syncwarp();
       continue;
     }
     P.cps = (uint32_t)prm[GTS_P_CTAS_PER_SM];
-    if (flags & GTS_FULL_TRACE) {
-      P.st = d_start + (size_t)q * g.row_nodes;
-      P.fi = d_finish + (size_t)q * g.row_nodes;
-    } else {
-      P.st = scratch + (size_t)gw * 2 * g.row_nodes;
-      P.fi = P.st + g.row_nodes;
-    }
+    P.st = (flags & GTS_FULL_TRACE) ? d_start + (size_t)q * g.row_nodes : nullptr;
+    P.fi = (flags & GTS_FULL_TRACE) ? d_finish + (size_t)q * g.row_nodes : nullptr;
+    P.scr = scratch + (size_t)gw * ((g.row_nodes + 1u) & ~1u);
     int32_t *cta_sm_row = (flags & GTS_WANT_CTA_SM) ? d_cta_sm + (size_t)q * g.row_ctas : nullptr;
 
     // ---- clear state
+    if (lane < (int)RC_N) {
+      uint32_t off = 0;
+      for (int r = 0; r < lane; r++) off += (uint32_t)prm[GTS_P_CAP_TENSOR + r];
+      sp[O_CAP + lane] = (uint32_t)prm[GTS_P_CAP_TENSOR + lane];
+      sp[O_OFF + lane] = off;
+      // the five rates sit at parameter indices 2, 4, 6, 8, 10 (HBM, TMA, SMEM, MMA, ALU)
+      *reinterpret_cast<uint64_t *>(sp + O_MAG + 2 * lane) = div_const((uint32_t)prm[GTS_P_HBM_BPC + 2 * lane]);
+    }
     for (uint32_t i = lane; i < P.L.S; i += 32) {
       sp[P.L.o_hid + i] = NONE;
       sp[P.L.o_key + i] = INF;
+      sp[P.L.o_meta + i] = RC_NONE;
+    }
+    for (uint32_t s = lane; s < P.L.NS; s += 32) {
+      uint32_t *o = sp + P.L.o_sm + s * SM_WORDS;
+      o[0] = INF; o[1] = NONE; o[2] = 0; o[3] = INF; o[4] = NONE; o[5] = 0;
     }
     for (uint32_t j = lane; j < P.L.Scta; j += 32) sp[P.L.o_cid + j] = NONE;
     for (uint32_t k = lane; k < P.L.NS * P.L.SC; k += 32) sp[P.L.o_sv + k] = 0u;
     for (uint32_t k = lane; k < P.L.cap_hbm; k += 32) sp[P.L.o_hs + k] = 0u;
-    for (uint32_t v = lane; v < nG; v += 32) P.st[v] = -1;
+    {
+      uint4 *z = reinterpret_cast<uint4 *>(P.scr);
+      const uint32_t nz = nG / 2;
+      for (uint32_t k = lane; k < nz; k += 32) z[k] = make_uint4(0, 0, 0, 0);
+      if ((nG & 1u) && lane == 0) P.scr[nG - 1] = make_uint2(0, 0);
+    }
     if (cta_sm_row)
       for (uint32_t c = lane; c < CG; c += 32) cta_sm_row[c] = -1;
+    __threadfence();
     __syncwarp();
 
-    const uint64_t step_limit = 8ull * nG + 4ull * CG + 64ull;
-    uint64_t steps = 0;
-    uint32_t next_cta = P.c0, issued = 0;
-    int32_t t = 0, mk = 0;
-    uint32_t H = 0;  // earliest free HBM server
+    Clock C;
+    C.t = 0;
+    C.H = 0;
+    C.next_ret = INF;
+    C.next_cta = P.c0;
+    C.steps = 0;
+    C.limit = 8ull * nG + 4ull * CG + 64ull;
+    uint32_t issued = 0;
+    int32_t mk = 0;
     uint64_t digest = 0;
-    bool ok = launch_ctas(g, P, t, next_cta, steps, step_limit, cta_sm_row, lane);
-    if (!ok) status = GTS_ERR_STEP_LIMIT;
+    Summary b{INF, NONE, 0};
+    if (!launch_ctas(g, P, C, cta_sm_row, lane, b)) status = GTS_ERR_STEP_LIMIT;
 
-    while (status == GTS_OK) {
-      // ---- issue, lowest id first, until nothing is issuable at t
-      for (;;) {
-        const bool hbm_ok = H <= (uint32_t)t;
-        uint32_t best = NONE, bslot = 0;
-        for (uint32_t i = lane; i < P.L.S; i += 32) {
-          if (sp[P.L.o_key + i] <= (uint32_t)t) {
-            const uint32_t h = sp[P.L.o_hid + i];
-            if (!(h & HBM_BIT) || hbm_ok) {
-              const uint32_t id = h & ID_MASK;
-              if (id < best) { best = id; bslot = i; }
-            }
+    while (status == GTS_OK && issued < nG) {
+      // ---- next event: lexicographic min of (effective cycle, node id) over all heads
+      const uint32_t E = __reduce_min_sync(FULL, b.k);
+      const uint32_t v = __reduce_min_sync(FULL, b.k == E ? b.id : NONE);
+      if (E > C.t) {
+        const uint32_t tn = min(E, C.next_ret);
+        if (tn == INF) { status = GTS_ERR_DEADLOCK; break; }
+        if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
+        C.t = tn;
+        if (C.next_ret <= C.t && !launch_ctas(g, P, C, cta_sm_row, lane, b)) { status = GTS_ERR_STEP_LIMIT; break; }
+        continue;
+      }
+      // ---- issue v, the lowest-id issuable head, at cycle t (all lanes, same values)
+      if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
+      const uint32_t owner = __ffs(__ballot_sync(FULL, b.k == E && b.id == v)) - 1;
+      const uint32_t i = __shfl_sync(FULL, b.sl, owner);
+      const uint32_t t = C.t;
+      const uint32_t cs = i / P.W;
+      const uint32_t sm = cs / P.cps;
+      const uint32_t hidv = sp[P.L.o_hid + i];
+      const uint32_t meta = sp[P.L.o_meta + i];
+      const uint32_t nx = sp[P.L.o_nxt + i];
+      const uint32_t sb = sp[P.L.o_sb + i];
+      const uint32_t cls = meta & 7u;
+      // one round of independent loads: the issued node's record, the next
+      // head's record, range and counters, and the successor entries
+      const uint4 rv = g.rec[v];
+      uint4 rn = make_uint4(0, 0, 0, 0), qn = rn;
+      uint2 cn = make_uint2(0, 0);
+      if (nx != NONE) {
+        rn = g.rec[nx];
+        qn = g.rng[nx];
+        if (lane == 0) cn = ld_counters(P.scr + (nx - P.n0));
+      }
+      uint32_t deg = (meta >> 3) & 31u;
+      if (deg == DEG_BIG) deg = g.rng[v].w - sb;
+      uint2 ew = make_uint2(NONE, 0);
+      if ((uint32_t)lane < deg) ew = g.succ[sb + lane];
+      cn.x = __shfl_sync(FULL, cn.x, 0);
+      cn.y = __shfl_sync(FULL, cn.y, 0);
+      uint32_t occ, hocc;
+      uint64_t lat;
+      node_cost(sp, rv.w & 15u, rv.x, rv.y, occ, hocc, lat);
+      const uint64_t f64 = (uint64_t)t + lat;
+      if (f64 > 0x7FFFFFFFull) { status = GTS_ERR_OVERFLOW; break; }
+      const uint32_t f = (uint32_t)f64;
+      __syncwarp();
+      // take one free server of the node's class on its SM (lane k tests server k)
+      if (cls != RC_NONE) {
+        uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + sp[O_OFF + cls];
+        const bool fr = (uint32_t)lane < sp[O_CAP + cls] && sv[lane] <= t;
+        const uint32_t bal = __ballot_sync(FULL, fr);
+        if (lane == __ffs(bal) - 1) sv[lane] = t + occ;
+      }
+      // take one free global HBM server
+      const uint32_t prevH = C.H;
+      if (hidv & HBM_BIT) {
+        uint32_t *hs = sp + P.L.o_hs;
+        const bool in = (uint32_t)lane < P.L.cap_hbm;
+        uint32_t hv = in ? hs[lane] : INF;
+        const uint32_t bal = __ballot_sync(FULL, in && hv <= t);
+        if (lane == __ffs(bal) - 1) {
+          hv = t + hocc;
+          hs[lane] = hv;
+        }
+        C.H = __reduce_min_sync(FULL, hv);
+      }
+      if (lane == 0) {
+        if (P.st) {
+          P.st[v - P.n0] = (int32_t)t;
+          P.fi[v - P.n0] = (int32_t)f;
+        }
+        if (want_digest) digest += mix64(((uint64_t)(v - P.n0) << 32 | t) ^ ((uint64_t)f * 0x9E3779B97F4A7C15ull));
+      }
+      const uint32_t rem = sp[P.L.o_crem + cs] - 1u;
+      const uint32_t cend = max(sp[P.L.o_cend + cs], f);
+      const uint32_t myc = sp[P.L.o_cid + cs];
+      __syncwarp();
+      sp[P.L.o_crem + cs] = rem;
+      sp[P.L.o_cend + cs] = cend;
+      mk = max(mk, (int32_t)f);
+      issued++;
+      // ---- release successors, in edge order
+      uint32_t adj_cnt = 0, adj_rdy = 0;
+      for (uint32_t base = 0; base < deg; base += 32) {
+        if (base) ew = (base + lane < deg) ? g.succ[sb + base + lane] : make_uint2(NONE, 0);
+        const uint32_t cnt = min(32u, deg - base);
+        for (uint32_t j = 0; j < cnt; j++) {
+          const uint32_t w = __shfl_sync(FULL, ew.x, j);
+          const uint32_t y = __shfl_sync(FULL, ew.y, j);
+          const uint32_t rel = (y & 1u) ? t : f;
+          if (w == nx) {  // the stream's next node becomes the head right below
+            adj_cnt++;
+            adj_rdy = max(adj_rdy, rel);
+            continue;
           }
-        }
-        const uint32_t v = __reduce_min_sync(FULL, best);
-        if (v == NONE) break;
-        const uint32_t owner = __ffs(__ballot_sync(FULL, best == v)) - 1;
-        const uint32_t i = __shfl_sync(FULL, bslot, owner);
-        if (++steps > step_limit) { status = GTS_ERR_STEP_LIMIT; break; }
-        const uint32_t lat = sp[P.L.o_L + i];
-        const int64_t f64 = (int64_t)t + (int64_t)lat;
-        if (f64 > 0x7FFFFFFFll) { status = GTS_ERR_OVERFLOW; break; }
-        const int32_t f = (int32_t)f64;
-        const uint32_t hid = sp[P.L.o_hid + i];
-        const uint32_t cls = sp[P.L.o_meta + i] & 7u;
-        const uint32_t cs = i / P.W;
-        const uint32_t sm = cs / P.cps;
-        // take one server of the node's per-SM class
-        if (cls != RC_NONE) {
-          uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + P.L.off[cls];
-          const uint32_t occ = sp[P.L.o_occ + i];
-          for (uint32_t b = 0; b < P.L.cap[cls]; b += 32) {
-            const uint32_t k = b + lane;
-            const bool fr = k < P.L.cap[cls] && sv[k] <= (uint32_t)t;
-            const uint32_t bal = __ballot_sync(FULL, fr);
-            if (bal) {
-              if (lane == (int)(__ffs(bal) - 1)) sv[k] = (uint32_t)t + occ;
-              break;
-            }
-          }
-        }
-        // take one global HBM server
-        if (hid & HBM_BIT) {
-          uint32_t *hs = sp + P.L.o_hs;
-          const uint32_t hocc = sp[P.L.o_hocc + i];
-          for (uint32_t b = 0; b < P.L.cap_hbm; b += 32) {
-            const uint32_t k = b + lane;
-            const bool fr = k < P.L.cap_hbm && hs[k] <= (uint32_t)t;
-            const uint32_t bal = __ballot_sync(FULL, fr);
-            if (bal) {
-              if (lane == (int)(__ffs(bal) - 1)) hs[k] = (uint32_t)t + hocc;
-              break;
-            }
-          }
-          __syncwarp();
-          uint32_t hm = INF;
-          for (uint32_t k = lane; k < P.L.cap_hbm; k += 32) hm = min(hm, hs[k]);
-          H = __reduce_min_sync(FULL, hm);
-        }
-        const uint32_t vl = v - P.n0;
-        if (lane == 0) {
-          P.st[vl] = t;
-          P.fi[vl] = f;
-          sp[P.L.o_crem + cs] -= 1u;
-          sp[P.L.o_cend + cs] = (uint32_t)max((int32_t)sp[P.L.o_cend + cs], f);
-          digest += mix64(((uint64_t)vl << 32 | (uint32_t)t) ^ ((uint64_t)(uint32_t)f * 0x9E3779B97F4A7C15ull));
-        }
-        mk = max(mk, f);
-        issued++;
-        // release successors that are warp heads right now
-        const uint32_t sb = sp[P.L.o_sb + i], se = sp[P.L.o_se + i];
-        const uint32_t myc = sp[P.L.o_cid + cs];
-        for (uint32_t e = sb + lane; e < se; e += 32) {
-          const uint2 s = g.succ[e];
-          const uint32_t wc = s.y >> 8;
+          const uint32_t wc = y >> 8;
           uint32_t tcs = NONE;
           if (wc == myc) {
             tcs = cs;
           } else {
-            for (uint32_t j = 0; j < P.L.Scta; j++)
-              if (sp[P.L.o_cid + j] == wc) { tcs = j; break; }
+            for (uint32_t jj = 0; jj < P.L.Scta; jj++)
+              if (sp[P.L.o_cid + jj] == wc) { tcs = jj; break; }
           }
-          if (tcs != NONE) {
-            const uint32_t j = tcs * P.W + ((s.y >> 1) & 127u);
-            if ((sp[P.L.o_hid + j] & ID_MASK) == s.x) {
-              atomicSub(&sp[P.L.o_np + j], 1u);
-              atomicMax(reinterpret_cast<int *>(&sp[P.L.o_rdy + j]), (s.y & 1u) ? t : f);
-            }
+          const uint32_t js = tcs * P.W + ((y >> 1) & 127u);
+          const bool head = tcs != NONE && (sp[P.L.o_hid + js] & ID_MASK) == w;
+          if (head) {
+            const uint32_t m2 = sp[P.L.o_meta + js] - 256u;
+            const uint32_t r2 = max(sp[P.L.o_rdy + js], rel);
+            __syncwarp();
+            sp[P.L.o_meta + js] = m2;
+            sp[P.L.o_rdy + js] = r2;
+            __syncwarp();
+          } else if (lane == 0) {
+            uint2 *c = P.scr + (w - P.n0);
+            atomicAdd(&c->x, 1u);
+            atomicMax(&c->y, rel);
           }
         }
+      }
+      set_head(P, i, nx, rn, qn, cn, adj_cnt, adj_rdy);
+      __syncwarp();
+      // ---- refresh keys and summaries the issue may have changed
+      if (g.cross_cta) {
+        for (uint32_t k = lane; k < P.L.S; k += 32) sp[P.L.o_key + k] = slot_key(P, k, t);
         __syncwarp();
-        // the stream advances to its next node
-        load_head_warp(g, P, i, sp[P.L.o_next + i], lane);
+        for (uint32_t s = lane; s < P.L.NS; s += 32) sm_summary(P, s, C.H);
+        b = lane_summary(P, lane);
+      } else {
+        const uint32_t k0 = sm * P.L.per;
+        for (uint32_t k = k0 + lane; k < min(k0 + P.L.per, P.L.S); k += 32) sp[P.L.o_key + k] = slot_key(P, k, t);
         __syncwarp();
-        // refresh the keys the issue may have changed
-        if (g.cross_cta) {
-          for (uint32_t k = lane; k < P.L.S; k += 32) sp[P.L.o_key + k] = slot_key(P, k);
+        if (C.H != prevH) {
+          for (uint32_t s = lane; s < P.L.NS; s += 32) sm_summary(P, s, C.H);
+          b = lane_summary(P, lane);
+        } else if ((uint32_t)lane == (sm & 31u)) {
+          sm_summary(P, sm, C.H);
+          b = lane_summary(P, lane);
+        }
+      }
+      __syncwarp();
+      if (rem == 0u) {
+        if (cend <= t) {
+          if (!launch_ctas(g, P, C, cta_sm_row, lane, b)) { status = GTS_ERR_STEP_LIMIT; break; }
         } else {
-          const uint32_t per = P.cps * P.W;
-          const uint32_t k0 = sm * per, k1 = min(k0 + per, P.L.S);
-          for (uint32_t k = k0 + lane; k < k1; k += 32) sp[P.L.o_key + k] = slot_key(P, k);
+          C.next_ret = min(C.next_ret, cend);
         }
-        __syncwarp();
-        if (sp[P.L.o_crem + cs] == 0u && (int32_t)sp[P.L.o_cend + cs] <= t) {
-          if (!launch_ctas(g, P, t, next_cta, steps, step_limit, cta_sm_row, lane)) {
-            status = GTS_ERR_STEP_LIMIT;
-            break;
-          }
-        }
-      }
-      if (status != GTS_OK || issued == nG) break;
-      // ---- advance to the next event cycle
-      uint32_t tn = INF;
-      for (uint32_t k = lane; k < P.L.S; k += 32) {
-        uint32_t key = sp[P.L.o_key + k];
-        if (key != INF) {
-          if (sp[P.L.o_hid + k] & HBM_BIT) key = max(key, H);
-          tn = min(tn, key);
-        }
-      }
-      for (uint32_t j = lane; j < P.L.Scta; j += 32) {
-        if (sp[P.L.o_cid + j] != NONE && sp[P.L.o_crem + j] == 0u) {
-          const uint32_t ce = sp[P.L.o_cend + j];
-          if (ce > (uint32_t)t) tn = min(tn, ce);
-        }
-      }
-      tn = __reduce_min_sync(FULL, tn);
-      if (tn == INF) { status = GTS_ERR_DEADLOCK; break; }
-      if (++steps > step_limit) { status = GTS_ERR_STEP_LIMIT; break; }
-      t = (int32_t)tn;
-      if (!launch_ctas(g, P, t, next_cta, steps, step_limit, cta_sm_row, lane)) {
-        status = GTS_ERR_STEP_LIMIT;
-        break;
       }
     }
     if (lane == 0) {
       d_status[q] = status;
       d_makespan[q] = status == GTS_OK ? mk : 0;
-      if (d_digest) d_digest[q] = status == GTS_OK ? digest : 0ull;
+      if (want_digest) d_digest[q] = status == GTS_OK ? digest : 0ull;
     }
     __syncwarp();
   }
@@ -561,7 +658,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
 size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct WsLayout {
-  size_t rec, rng, succ, pred, first, cnt, noff, coff, total;
+  size_t rec, rng, succ, first, cnt, noff, coff, total;
 };
 
 bool ws_layout(uint64_t n, uint64_t m, uint64_t C, uint64_t W, uint64_t G, WsLayout &w) {
@@ -570,7 +667,6 @@ bool ws_layout(uint64_t n, uint64_t m, uint64_t C, uint64_t W, uint64_t G, WsLay
   w.rec = o; o += align_up(n * 16);
   w.rng = o; o += align_up(n * 16);
   w.succ = o; o += align_up(m * 8);
-  w.pred = o; o += align_up(m * 4);
   w.first = o; o += align_up(C * W * 4);
   w.cnt = o; o += align_up(C * 4);
   w.noff = o; o += align_up((G + 1) * 4);
@@ -694,15 +790,11 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   }
 
   // ---- derived arrays
-  std::vector<uint32_t> indeg(n + 1, 0), pptr(n + 1, 0), pred(m), first(C * W, NONE), nxt(n, NONE), cnt(C, 0);
+  std::vector<uint32_t> indeg(n, 0), first(C * W, NONE), nxt(n, NONE), cnt(C, 0);
   for (uint64_t x = 0; x < m; x++) indeg[col[x]]++;
-  for (uint64_t v = 0; v < n; v++) pptr[v + 1] = pptr[v] + indeg[v];
-  {
-    std::vector<uint32_t> cur(pptr.begin(), pptr.end() - 1);
-    for (uint64_t u = 0; u < n; u++)
-      for (uint32_t x = row_ptr[u]; x < row_ptr[u + 1]; x++)
-        pred[cur[col[x]]++] = (uint32_t)u | ((uint32_t)ek[x] << 31);
-  }
+  for (uint64_t v = 0; v < n; v++)
+    if (indeg[v] > MAX_INDEG)
+      return fail(GTS_ERR_UNSUPPORTED, "node " + std::to_string(v) + " has more than 2^24-1 predecessors");
   for (uint64_t v = n; v-- > 0;) {
     const uint64_t key = (uint64_t)cta[v] * W + wp[v];
     nxt[v] = first[key];
@@ -711,8 +803,8 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   for (uint64_t v = 0; v < n; v++) cnt[cta[v]]++;
   std::vector<uint4> rec(n), rng(n);
   for (uint64_t v = 0; v < n; v++) {
-    rec[v] = make_uint4(work[v], lx[v], nxt[v], (uint32_t)ty[v] | ((uint32_t)wp[v] << 4));
-    rng[v] = make_uint4(pptr[v], pptr[v + 1], row_ptr[v], row_ptr[v + 1]);
+    rec[v] = make_uint4(work[v], lx[v], nxt[v], (uint32_t)ty[v] | (indeg[v] << 4));
+    rng[v] = make_uint4(0u, 0u, row_ptr[v], row_ptr[v + 1]);
   }
   std::vector<uint2> succ(m);
   for (uint64_t x = 0; x < m; x++)
@@ -726,7 +818,6 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   up(wl.rec, rec.data(), n * 16);
   up(wl.rng, rng.data(), n * 16);
   up(wl.succ, succ.data(), m * 8);
-  up(wl.pred, pred.data(), m * 4);
   up(wl.first, first.data(), C * W * 4);
   up(wl.cnt, cnt.data(), C * 4);
   up(wl.noff, noff.data(), (G + 1) * 4);
@@ -744,7 +835,6 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   dg.rec = (const uint4 *)(ws + wl.rec);
   dg.rng = (const uint4 *)(ws + wl.rng);
   dg.succ = (const uint2 *)(ws + wl.succ);
-  dg.pred = (const uint32_t *)(ws + wl.pred);
   dg.stream_first = (const uint32_t *)(ws + wl.first);
   dg.cta_cnt = (const uint32_t *)(ws + wl.cnt);
   dg.cta_kernel = d->cta_kernel;
@@ -797,34 +887,52 @@ gts_status gts_params_destroy(gts_params *p) {
 }
 
 namespace {
+// Per-warp scratch: one (released-predecessor count, max release cycle) pair
+// per node of the largest graph, rounded to 16 bytes.
+uint64_t scratch_row_bytes(const gts_graph *g) { return (((uint64_t)g->dg.row_nodes + 1) & ~1ull) * 8; }
+
 struct Plan {
   uint32_t words, wpb, smem, blocks, warps;
 };
 
 gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, uint32_t np, uint32_t flags,
                        size_t scratch_bytes, bool limit_by_scratch, Plan &pl) {
+  (void)flags;
   uint32_t words = 64;
   for (uint32_t p = first; p < first + np; p++) words = std::max(words, P->words[p]);
   const uint32_t bytes = words * 4;
   pl.words = words;
-  pl.wpb = std::max(1u, std::min((uint32_t)MAX_WPB, MAX_SMEM_BYTES / bytes));
-  pl.smem = pl.wpb * bytes;
-  cudaError_t e = cudaFuncSetAttribute(k_simulate, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem);
-  if (e != cudaSuccess) return cuda_fail(e, "simulate: set shared memory size");
-  int nb = 0, dev = 0, sms = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_simulate, (int)pl.wpb * 32, pl.smem);
+  cudaError_t e = cudaFuncSetAttribute(k_simulate, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)MAX_SMEM_BYTES);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_simulate, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e != cudaSuccess) return cuda_fail(e, "simulate: occupancy query");
-  uint64_t warps = (uint64_t)std::max(nb, 1) * sms * pl.wpb;
+  if (e != cudaSuccess) return cuda_fail(e, "simulate: kernel attributes");
+  // warps per block: whichever keeps the most design points resident per SM
+  uint32_t best_w = 0;
+  pl.wpb = 1;
+  for (uint32_t wpb = MAX_WPB; wpb >= 1; wpb /= 2) {
+    if (wpb * bytes > MAX_SMEM_BYTES) continue;
+    int nb = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_simulate, (int)wpb * 32, wpb * bytes);
+    if (e != cudaSuccess) return cuda_fail(e, "simulate: occupancy query");
+    if ((uint32_t)nb * wpb > best_w) {
+      best_w = (uint32_t)nb * wpb;
+      pl.wpb = wpb;
+    }
+  }
+  pl.smem = pl.wpb * bytes;
+  uint64_t warps = (uint64_t)std::max(best_w, 1u) * sms;
   warps = std::min<uint64_t>(warps, np);
-  if (limit_by_scratch && !(flags & GTS_FULL_TRACE)) {
-    const uint64_t row = (uint64_t)g->dg.row_nodes * 8;
-    const uint64_t fit = row ? scratch_bytes / row : warps;
-    if (fit == 0) return fail(GTS_ERR_NOMEM, "scratch smaller than one point's start/finish rows");
+  if (limit_by_scratch) {
+    const uint64_t row = scratch_row_bytes(g);
+    const uint64_t fit = scratch_bytes / row;
+    if (fit == 0) return fail(GTS_ERR_NOMEM, "scratch smaller than one design point's counter row");
     warps = std::min(warps, fit);
   }
   pl.warps = (uint32_t)std::max<uint64_t>(warps, 1);
+  pl.wpb = std::min(pl.wpb, pl.warps);
+  pl.smem = pl.wpb * bytes;
   pl.blocks = (pl.warps + pl.wpb - 1) / pl.wpb;
   return GTS_OK;
 }
@@ -832,10 +940,9 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
 
 size_t gts_scratch_bytes(const gts_graph *g, const gts_params *P, uint32_t flags) {
   if (!g || !P) return 0;
-  if (flags & GTS_FULL_TRACE) return 0;
   Plan pl;
   if (plan_launch(g, P, 0, P->n_points, flags, 0, false, pl) != GTS_OK) return 0;
-  return (size_t)pl.warps * g->dg.row_nodes * 8;
+  return (size_t)pl.warps * scratch_row_bytes(g);
 }
 
 gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point, uint32_t n_points, uint32_t flags,
@@ -848,10 +955,12 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
   if (flags & ~(GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM)) return fail(GTS_ERR_INVALID_ARG, "unknown flag");
   if ((uint64_t)first_point + n_points > P->n_points) return fail(GTS_ERR_INVALID_ARG, "point range outside the table");
   if (!d_makespan || !d_status) return fail(GTS_ERR_INVALID_ARG, "d_makespan and d_status are required");
-  if ((flags & GTS_FULL_TRACE) && (!d_start || !d_finish)) return fail(GTS_ERR_INVALID_ARG, "FULL_TRACE needs d_start and d_finish");
+  if ((flags & GTS_FULL_TRACE) && g->dg.row_nodes && (!d_start || !d_finish))
+    return fail(GTS_ERR_INVALID_ARG, "FULL_TRACE needs d_start and d_finish");
   if ((flags & GTS_WANT_DIGEST) && !d_digest) return fail(GTS_ERR_INVALID_ARG, "WANT_DIGEST needs d_digest");
-  if ((flags & GTS_WANT_CTA_SM) && !d_cta_sm) return fail(GTS_ERR_INVALID_ARG, "WANT_CTA_SM needs d_cta_sm");
-  if (!(flags & GTS_FULL_TRACE) && !d_scratch && g->dg.row_nodes) return fail(GTS_ERR_NOMEM, "scratch required without FULL_TRACE");
+  if ((flags & GTS_WANT_CTA_SM) && g->dg.row_ctas && !d_cta_sm) return fail(GTS_ERR_INVALID_ARG, "WANT_CTA_SM needs d_cta_sm");
+  if (!d_scratch) return fail(GTS_ERR_NOMEM, "scratch required (gts_scratch_bytes)");
+  if ((uintptr_t)d_scratch % 16 != 0) return fail(GTS_ERR_INVALID_ARG, "scratch must be 16-byte aligned");
   cudaStream_t s = (cudaStream_t)stream;
   if (n_points) {
     Plan pl;
@@ -860,7 +969,7 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
     k_simulate<<<pl.blocks, pl.wpb * 32, pl.smem, s>>>(
         g->dg, P->d_params, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status,
         (flags & GTS_WANT_DIGEST) ? d_digest : nullptr, (flags & GTS_WANT_CTA_SM) ? d_cta_sm : nullptr,
-        (int32_t *)d_scratch, pl.warps, pl.words);
+        (uint2 *)d_scratch, pl.warps, pl.words);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "simulate: launch");
   }

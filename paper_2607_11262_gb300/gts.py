@@ -159,6 +159,14 @@ def gts_last_error():
 
 
 # ---------------------------------------------------------------- torch-owned buffers
+class _null:
+    def __enter__(self):
+        return None
+
+    def __exit__(self, *a):
+        return False
+
+
 def _stream_handle(stream):
     import torch
     if stream is None:
@@ -169,7 +177,12 @@ def _stream_handle(stream):
 class DeviceGraph:
     """A workloads.Graph resident on the GPU, validated and packed by libgts."""
 
-    def __init__(self, graph, device="cuda", stream=None):
+    FIELDS = ("row_ptr", "col", "ekind", "type", "warp", "cta", "work", "lat_extra", "cta_kernel",
+              "node_off", "cta_off")
+
+    def __init__(self, graph, device="cuda", stream=None, tensors=None):
+        """``tensors`` (optional): the graph's arrays already on the device,
+        keyed like FIELDS (uint32 arrays as int32, uint16 as int16)."""
         import torch
         self.graph = graph
         dev = torch.device(device)
@@ -181,14 +194,17 @@ class DeviceGraph:
             elif a.dtype == np.uint16:
                 a = a.view(np.int16)
             return torch.from_numpy(a).to(dev)
-        self.tensors = {k: t(getattr(graph, k)) for k in
-                        ("row_ptr", "col", "ekind", "type", "warp", "cta", "work", "lat_extra", "cta_kernel",
-                         "node_off", "cta_off")}
+        if tensors is None:
+            tensors = {k: t(getattr(graph, k)) for k in self.FIELDS}
+        else:
+            dev = next(iter(tensors.values())).device
+        self.tensors = tensors
         n, m, C, W, G = graph.n_nodes, graph.n_edges, graph.n_ctas, graph.warps_per_cta, graph.n_graphs
         nbytes = gts_graph_workspace_bytes(n, m, C, W, G)
         if nbytes == 0:
             raise GtsError(GTS_ERR_INVALID_ARG, "graph size out of range")
-        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        with torch.cuda.stream(stream) if stream is not None else _null():
+            self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
         T = self.tensors
         d = GraphDesc(n, m, C, W, G, T["node_off"].data_ptr(), T["cta_off"].data_ptr(), T["row_ptr"].data_ptr(),
                       T["col"].data_ptr(), T["ekind"].data_ptr(), T["type"].data_ptr(), T["warp"].data_ptr(),
@@ -198,6 +214,10 @@ class DeviceGraph:
         self.handle = gts_graph_create(d, _stream_handle(stream))
         self.row_nodes = gts_row_nodes(self.handle)
         self.row_ctas = gts_row_ctas(self.handle)
+
+    @classmethod
+    def from_device_tensors(cls, graph, tensors, stream=None):
+        return cls(graph, stream=stream, tensors=tensors)
 
     def close(self):
         if getattr(self, "handle", None):
@@ -214,13 +234,21 @@ class DeviceGraph:
 class DeviceParams:
     """A [P][24] int32 parameter table resident on the GPU."""
 
-    def __init__(self, dgraph: DeviceGraph, params, stream=None):
+    def __init__(self, dgraph: DeviceGraph, params, stream=None, tensor=None, n_points=None):
         import torch
         self.dgraph = dgraph
-        p = np.ascontiguousarray(params, np.int32)
-        self.n_points = int(p.shape[0])
-        self.tensor = torch.from_numpy(p.reshape(-1)).to(dgraph.workspace.device)
+        if tensor is None:
+            p = np.ascontiguousarray(params, np.int32)
+            self.n_points = int(p.shape[0])
+            self.tensor = torch.from_numpy(p.reshape(-1)).to(dgraph.workspace.device)
+        else:
+            self.n_points = int(n_points)
+            self.tensor = tensor
         self.handle = gts_params_upload(dgraph.handle, self.tensor.data_ptr(), self.n_points, _stream_handle(stream))
+
+    @classmethod
+    def from_device_tensor(cls, dgraph, tensor, n_points, stream=None):
+        return cls(dgraph, None, stream=stream, tensor=tensor, n_points=n_points)
 
     def close(self):
         if getattr(self, "handle", None):
@@ -272,7 +300,7 @@ def simulate(dgraph: DeviceGraph, dparams: DeviceParams, first_point=0, n_points
         n_points = dparams.n_points - first_point
     if out is None:
         out = alloc_outputs(dgraph, n_points, flags)
-    if scratch is None and not (flags & GTS_FULL_TRACE):
+    if scratch is None:
         nb = gts_scratch_bytes(dgraph.handle, dparams.handle, flags)
         scratch = torch.empty(max(nb, 16), dtype=torch.uint8, device=dgraph.workspace.device)
     gts_simulate_batch(dgraph.handle, dparams.handle, first_point, n_points, flags, _ptr(out.start),

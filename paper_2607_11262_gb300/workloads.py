@@ -465,18 +465,23 @@ def gemm512() -> Graph:
     return assemble("gemm512", 4, [tpl], np.zeros(16, np.int64), np.zeros(16, np.uint32))
 
 
-def wsgemm8192(num_ctas=132) -> Graph:
-    """Warp-specialised persistent GEMM M=N=K=8192 bf16, 128x256x64 tiles.
+def ws_gemm(M=8192, N=8192, K=8192, num_ctas=132, name="wsgemm8192") -> Graph:
+    """Warp-specialised persistent GEMM (bf16, 128x256x64 tiles).
 
-    2048 output tiles over ``num_ctas`` persistent CTAs (tile t -> CTA t mod
-    num_ctas), 4-stage ring, 128 k-steps per tile.
+    (M/128)*(N/256) output tiles over ``num_ctas`` persistent CTAs (tile t ->
+    CTA t mod num_ctas), 4-stage ring, K/64 k-steps per tile.
     """
-    tiles = (8192 // 128) * (8192 // 256)
+    tiles = (M // 128) * (N // 256)
     per = np.array([tiles // num_ctas + (1 if c < tiles % num_ctas else 0) for c in range(num_ctas)])
     kinds = sorted(set(per.tolist()), reverse=True)
-    tpls = [ws_gemm_cta(k, 8192 // 64) for k in kinds]
+    tpls = [ws_gemm_cta(k, K // 64) for k in kinds]
     ct = np.array([kinds.index(x) for x in per], np.int64)
-    return assemble("wsgemm8192", 3, tpls, ct, np.zeros(num_ctas, np.uint32))
+    return assemble(name, 3, tpls, ct, np.zeros(num_ctas, np.uint32))
+
+
+def wsgemm8192(num_ctas=132) -> Graph:
+    """M=N=K=8192: 2048 tiles over 132 persistent CTAs, 128 k-steps per tile."""
+    return ws_gemm(8192, 8192, 8192, num_ctas)
 
 
 def fa_fwd(batch=4, heads=32, seq=4096, head_dim=128, q_block=128, kv_block=128) -> Graph:
@@ -646,6 +651,10 @@ def workload(name: str, points: int | None = None, instances: int | None = None)
         g = wsgemm8192()
         p = sweep_params(SEED0 + 2, 4096, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE], 1)
         d = "WS persistent GEMM 8192^3 bf16, 128x256x64, 1 producer + 2 consumer WGs, 4-stage ring, 132 CTAs; 4096 points"
+    elif name == "wsgemm_small":
+        g = ws_gemm(2048, 2048, 1024, 132, "wsgemm_small")
+        p = sweep_params(SEED0 + 2, 4096, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE], 1)
+        d = "WS GEMM 2048x2048x1024 (profiling-size case of the wsgemm8192 kernel shape); 4096 points"
     elif name == "fa_fwd":
         g = fa_fwd()
         p = sweep_params(SEED0 + 3, 1024, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE, AX_ALU_RATE], 1)

@@ -129,8 +129,8 @@ def test_makespan_only_with_tiny_scratch():
     w = W.workload("gemm512")
     dg = gts.DeviceGraph(w.graph)
     dp = gts.DeviceParams(dg, w.params)
-    row = dg.row_nodes * 8
-    scratch = torch.empty(3 * row, dtype=torch.uint8, device="cuda")  # 3 warps at a time
+    row = ((dg.row_nodes + 1) // 2 * 2) * 8
+    scratch = torch.empty(3 * row, dtype=torch.uint8, device="cuda")  # 3 design points at a time
     out = gts.simulate(dg, dp, flags=gts.GTS_WANT_DIGEST, scratch=scratch)
     torch.cuda.synchronize()
     full = H.run_gpu(w.graph, w.params)
