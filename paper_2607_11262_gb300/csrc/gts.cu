@@ -17,14 +17,14 @@
 //    server.  Every unissued head keeps effective cycle >= t (keys are clamped
 //    to the cycle they are computed at; a head that could issue at t but did
 //    not has had its key recomputed when its unit or H changed), so the next
-//    event is the lexicographic minimum of (effective cycle, node id) over
-//    all heads: if that cycle is t, the node is the lowest-id issuable head;
-//    otherwise it is the next event cycle.  Lane l owns simulated SMs
-//    l, l+32, ...; each SM keeps the (cycle, id) minimum of its non-HBM heads
-//    and of its HBM heads in shared memory, each lane the minimum over its SMs
-//    in registers, and the warp takes the minimum over lanes with two
-//    __reduce_min_sync.  After an issue only the issuing SM's owner lane
-//    recomputes (all lanes when H moved).
+//    event is the minimum of (effective cycle << 32 | node id) over all
+//    heads: if its cycle is t, the node is the lowest-id issuable head;
+//    otherwise it is the next event cycle.  Each simulated SM keeps that
+//    minimum over its heads; lane l owns SMs l, l+32, ... and keeps the
+//    minimum over them in registers; the warp takes the minimum over lanes
+//    with two __reduce_min_sync.  After an issue the issuing SM's keys and
+//    summary are recomputed warp-parallel, then its owner lane's minimum;
+//    when H moves, the SMs whose HBM heads it overtakes are recomputed.
 //  * The issue itself runs in every lane on broadcast values (no divergence);
 //    only global atomics and scratch-counter reads are lane 0's.
 //  * Dependency release (Section 5.1).  An issued node releases each
@@ -61,6 +61,7 @@ namespace {
 
 constexpr uint32_t NONE = 0xFFFFFFFFu;     // no node / no CTA
 constexpr uint32_t INF = 0xFFFFFFFFu;      // key of a head that cannot issue
+constexpr uint64_t INF64 = ~0ull;
 constexpr uint32_t HBM_BIT = 0x80000000u;  // on a slot's node id: node uses HBM
 constexpr uint32_t ID_MASK = 0x7FFFFFFFu;
 constexpr uint32_t FULL = 0xFFFFFFFFu;
@@ -72,8 +73,13 @@ constexpr uint32_t DEG_BIG = 31;            // successor count field: 31 = read 
 
 // per-SM resource classes (Section 5.2)
 enum : uint32_t { RC_TENSOR = 0, RC_TMA = 1, RC_LSU = 2, RC_ALU = 3, RC_BAR = 4, RC_N = 5, RC_NONE = 7 };
-// rates with a division constant
-enum : uint32_t { RT_HBM = 0, RT_TMA = 1, RT_SMEM = 2, RT_MMA = 3, RT_ALU = 4 };
+// Per node type (LOAD, SMEM, MMA, EW, STORE, BAR, NOP), one nibble each:
+// its per-SM class, and the rate that sets its occupancy (0 HBM, 1 TMA,
+// 2 SMEM, 3 MMA, 4 ALU, 5 = one cycle, 6 = none).  LOAD and STORE also take
+// an HBM server.
+constexpr uint32_t TYPE_CLASS = 0x7413021u;
+constexpr uint32_t TYPE_RATE = 0x6514321u;
+constexpr uint32_t TYPE_HBM = 0x11u;
 static_assert(GTS_P_TMA_BPC == GTS_P_HBM_BPC + 2 && GTS_P_SMEM_BPC == GTS_P_HBM_BPC + 4 &&
                   GTS_P_MMA_FMA_PC == GTS_P_HBM_BPC + 6 && GTS_P_ALU_OPS_PC == GTS_P_HBM_BPC + 8,
               "rate k of the division-constant table sits at parameter index GTS_P_HBM_BPC + 2k");
@@ -110,19 +116,24 @@ struct DevGraph {
 constexpr uint32_t O_CAP = GTS_NPARAM;       // 5 words: servers per class
 constexpr uint32_t O_OFF = GTS_NPARAM + 5;   // 5 words: class offset inside an SM's servers
 constexpr uint32_t O_MAG = GTS_NPARAM + 10;  // 5 x 2 words: division constants of the rates
-constexpr uint32_t O_DYN = GTS_NPARAM + 20;  // first per-point array (even: 8-byte aligned)
-constexpr uint32_t SM_WORDS = 6;             // per SM: lo key, lo id, lo slot, hbm key, hbm id, hbm slot
+constexpr uint32_t O_BASE = GTS_NPARAM + 20; // 8 words: base latency per node type
+constexpr uint32_t O_DYN = GTS_NPARAM + 28;  // first per-point array (16-byte aligned)
+// slot record (6 words): id|HBM, key, rdy, pending<<8 | deg<<3 | class, next, successor begin
+constexpr uint32_t F_HID = 0, F_KEY = 1, F_RDY = 2, F_META = 3, F_NXT = 4, F_SB = 5, SLOT_WORDS = 6;
+// SM record (4 words): best id, best effective cycle, best slot, min key of its HBM heads
+constexpr uint32_t SM_WORDS = 4;
+// CTA slot record (4 words): CTA id, nodes not issued, max finish, kernel
+constexpr uint32_t C_ID = 0, C_REM = 1, C_END = 2, C_KERN = 3, CTA_WORDS = 4;
 
 struct Layout {
   uint32_t S, Scta, NS, SC, cap_hbm, per;
-  uint32_t o_hid, o_key, o_rdy, o_meta, o_nxt, o_sb, o_sm, o_cid, o_crem, o_cend, o_ckern, o_sv, o_hs, words;
+  uint32_t o_slot, o_sm, o_cta, o_sv, o_hs, words;
 };
 
 __host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
   if (p[GTS_P_NUM_SMS] < 1 || p[GTS_P_CTAS_PER_SM] < 1) return GTS_ERR_INVALID_PARAMS;
-  const int rates[5] = {GTS_P_HBM_BPC, GTS_P_TMA_BPC, GTS_P_SMEM_BPC, GTS_P_MMA_FMA_PC, GTS_P_ALU_OPS_PC};
   for (int i = 0; i < 5; i++)
-    if (p[rates[i]] < 1) return GTS_ERR_INVALID_PARAMS;
+    if (p[GTS_P_HBM_BPC + 2 * i] < 1) return GTS_ERR_INVALID_PARAMS;
   const int lats[6] = {GTS_P_DRAM_LAT, GTS_P_TMA_LAT, GTS_P_SMEM_LAT, GTS_P_MMA_LAT, GTS_P_ALU_LAT, GTS_P_BAR_LAT};
   for (int i = 0; i < 6; i++)
     if (p[lats[i]] < 0) return GTS_ERR_INVALID_PARAMS;
@@ -156,17 +167,9 @@ __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint3
   if ((uint64_t)p[GTS_P_CAP_HBM] > 32) return false;
   L.cap_hbm = (uint32_t)p[GTS_P_CAP_HBM];
   uint64_t w = O_DYN;
-  L.o_hid = (uint32_t)w; w += L.S;
-  L.o_key = (uint32_t)w; w += L.S;
-  L.o_rdy = (uint32_t)w; w += L.S;
-  L.o_meta = (uint32_t)w; w += L.S;
-  L.o_nxt = (uint32_t)w; w += L.S;
-  L.o_sb = (uint32_t)w; w += L.S;
+  L.o_slot = (uint32_t)w; w += (uint64_t)L.S * SLOT_WORDS;
   L.o_sm = (uint32_t)w; w += (uint64_t)L.NS * SM_WORDS;
-  L.o_cid = (uint32_t)w; w += L.Scta;
-  L.o_crem = (uint32_t)w; w += L.Scta;
-  L.o_cend = (uint32_t)w; w += L.Scta;
-  L.o_ckern = (uint32_t)w; w += L.Scta;
+  L.o_cta = (uint32_t)w; w += (uint64_t)L.Scta * CTA_WORDS;
   L.o_sv = (uint32_t)w; w += (uint64_t)L.NS * L.SC;
   L.o_hs = (uint32_t)w; w += L.cap_hbm;
   w = (w + 3) & ~(uint64_t)3;  // 16-byte multiple
@@ -198,70 +201,51 @@ __device__ __forceinline__ uint2 ld_counters(const uint2 *p) {  // strong load o
   return r;
 }
 
+__device__ __forceinline__ uint64_t pack(uint32_t eff, uint32_t id) { return (uint64_t)eff << 32 | id; }
+
+// Warp-wide minimum of a u64 (all lanes get it) and the lowest lane holding it.
+__device__ __forceinline__ uint64_t warp_min64(uint64_t x, uint32_t &lane_of) {
+  const uint32_t hi = __reduce_min_sync(FULL, (uint32_t)(x >> 32));
+  const uint32_t lo = __reduce_min_sync(FULL, (uint32_t)(x >> 32) == hi ? (uint32_t)x : NONE);
+  const uint64_t m = pack(hi, lo);
+  lane_of = __ffs(__ballot_sync(FULL, x == m)) - 1;
+  return m;
+}
+
 struct Pt {
   uint32_t *sp;  // this warp's shared-memory words
   Layout L;
   uint32_t W, cps, n0, c0, c1;
   int32_t *st, *fi;  // trace rows (graph-local index) or null
   uint2 *scr;        // scratch counters (graph-local index)
+  __device__ __forceinline__ uint32_t *slot(uint32_t i) const { return sp + L.o_slot + i * SLOT_WORDS; }
+  __device__ __forceinline__ uint32_t *smrec(uint32_t s) const { return sp + L.o_sm + s * SM_WORDS; }
+  __device__ __forceinline__ uint32_t *cta(uint32_t j) const { return sp + L.o_cta + j * CTA_WORDS; }
 };
-
-// Per-SM class and HBM use of a node type (Section 4.1 operation descriptor).
-__device__ __forceinline__ uint32_t type_class(uint32_t type) {
-  switch (type) {
-    case GTS_LOAD: case GTS_STORE: return RC_TMA;
-    case GTS_SMEM: return RC_LSU;
-    case GTS_MMA: return RC_TENSOR;
-    case GTS_EW: return RC_ALU;
-    case GTS_BAR: return RC_BAR;
-    default: return RC_NONE;
-  }
-}
-__device__ __forceinline__ bool type_hbm(uint32_t type) { return type == GTS_LOAD || type == GTS_STORE; }
-
-__device__ __forceinline__ uint32_t rate_occ(const uint32_t *sp, uint32_t work, uint32_t rt, int pidx) {
-  const uint64_t M = *reinterpret_cast<const uint64_t *>(sp + O_MAG + 2 * rt);
-  return cdiv_c(work, sp[pidx], M);
-}
 
 // Occupancies and latency of a node (Section 5.2 throughput model).
 __device__ __forceinline__ void node_cost(const uint32_t *sp, uint32_t type, uint32_t work, uint32_t lx,
                                           uint32_t &occ, uint32_t &hocc, uint64_t &lat) {
-  uint32_t base = 0;
-  occ = 0;
-  hocc = 0;
-  switch (type) {
-    case GTS_LOAD:
-      occ = rate_occ(sp, work, RT_TMA, GTS_P_TMA_BPC);
-      hocc = rate_occ(sp, work, RT_HBM, GTS_P_HBM_BPC);
-      base = sp[GTS_P_TMA_LAT] + sp[GTS_P_DRAM_LAT];
-      break;
-    case GTS_SMEM: occ = rate_occ(sp, work, RT_SMEM, GTS_P_SMEM_BPC); base = sp[GTS_P_SMEM_LAT]; break;
-    case GTS_MMA: occ = rate_occ(sp, work, RT_MMA, GTS_P_MMA_FMA_PC); base = sp[GTS_P_MMA_LAT]; break;
-    case GTS_EW: occ = rate_occ(sp, work, RT_ALU, GTS_P_ALU_OPS_PC); base = sp[GTS_P_ALU_LAT]; break;
-    case GTS_STORE:
-      occ = rate_occ(sp, work, RT_TMA, GTS_P_TMA_BPC);
-      hocc = rate_occ(sp, work, RT_HBM, GTS_P_HBM_BPC);
-      base = sp[GTS_P_TMA_LAT];
-      break;
-    case GTS_BAR: occ = 1; base = sp[GTS_P_BAR_LAT]; break;
-    default: break;
-  }
-  lat = (uint64_t)base + lx + (occ > hocc ? occ : hocc);
+  const uint32_t rt = (TYPE_RATE >> (4 * type)) & 15u;
+  occ = rt == 5u ? 1u : 0u;
+  if (rt < 5u) occ = cdiv_c(work, sp[GTS_P_HBM_BPC + 2 * rt], *reinterpret_cast<const uint64_t *>(sp + O_MAG + 2 * rt));
+  hocc = 0u;
+  if ((TYPE_HBM >> type) & 1u) hocc = cdiv_c(work, sp[GTS_P_HBM_BPC], *reinterpret_cast<const uint64_t *>(sp + O_MAG));
+  lat = (uint64_t)sp[O_BASE + type] + lx + (occ > hocc ? occ : hocc);
 }
 
 // Key of slot i computed at cycle t (>= t; INF if it cannot issue yet).
 __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t) {
-  const uint32_t *sp = P.sp;
-  const uint32_t h = sp[P.L.o_hid + i];
-  const uint32_t meta = sp[P.L.o_meta + i];
+  const uint32_t *sl = P.slot(i);
+  const uint32_t h = sl[F_HID];
+  const uint32_t meta = sl[F_META];
   if (h == NONE || (meta >> 8) != 0u) return INF;
-  uint32_t k = max(sp[P.L.o_rdy + i], t);
+  uint32_t k = max(sl[F_RDY], t);
   const uint32_t cls = meta & 7u;
   if (cls != RC_NONE) {
     const uint32_t sm = i / P.L.per;
-    const uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + sp[O_OFF + cls];
-    const uint32_t cap = sp[O_CAP + cls];
+    const uint32_t *sv = P.sp + P.L.o_sv + sm * P.L.SC + P.sp[O_OFF + cls];
+    const uint32_t cap = P.sp[O_CAP + cls];
     uint32_t a = sv[0];
     for (uint32_t q = 1; q < cap; q++) a = min(a, sv[q]);
     k = max(k, a);
@@ -269,44 +253,95 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
   return k;
 }
 
-__device__ __forceinline__ bool lex_less(uint32_t k1, uint32_t id1, uint32_t k2, uint32_t id2) {
-  return k1 < k2 || (k1 == k2 && id1 < id2);
-}
-
-// Recomputes the summary of SM s from its slots' keys (one lane).
-__device__ void sm_summary(const Pt &P, uint32_t s, uint32_t H) {
-  uint32_t *sp = P.sp;
-  uint32_t lk = INF, lid = NONE, lsl = 0, hk = INF, hid = NONE, hsl = 0;
+// Warp-parallel: recompute (when `keys`) the keys of SM s's slots at cycle t
+// and its summary record.  All lanes call it.
+__device__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, bool keys, int lane) {
   const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
-  for (uint32_t i = i0; i < i1; i++) {
-    const uint32_t k = sp[P.L.o_key + i];
-    const uint32_t h = sp[P.L.o_hid + i];
-    if (k == INF) continue;
-    const uint32_t id = h & ID_MASK;
-    if (h & HBM_BIT) {
-      const uint32_t e = max(k, H);
-      if (lex_less(e, id, hk, hid)) { hk = e; hid = id; hsl = i; }
-    } else if (lex_less(k, id, lk, lid)) {
-      lk = k; lid = id; lsl = i;
+  uint64_t best = INF64;
+  uint32_t bsl = 0, hmin = INF;
+  for (uint32_t base = i0; base < i1; base += 32) {
+    const uint32_t i = base + lane;
+    uint64_t val = INF64;
+    if (i < i1) {
+      uint32_t *sl = P.slot(i);
+      const uint32_t k = keys ? slot_key(P, i, t) : sl[F_KEY];
+      if (keys) sl[F_KEY] = k;
+      const uint32_t h = sl[F_HID];
+      if (k != INF) {
+        const bool hb = (h & HBM_BIT) != 0u;
+        val = pack(hb ? max(k, H) : k, h & ID_MASK);
+        if (hb) hmin = min(hmin, k);
+      }
+    }
+    uint32_t who;
+    const uint64_t m = warp_min64(val, who);
+    if (m < best) {
+      best = m;
+      bsl = base + who;
     }
   }
-  uint32_t *o = sp + P.L.o_sm + s * SM_WORDS;
-  o[0] = lk; o[1] = lid; o[2] = lsl; o[3] = hk; o[4] = hid; o[5] = hsl;
+  hmin = __reduce_min_sync(FULL, hmin);
+  if (lane == 0) {
+    uint32_t *o = P.smrec(s);
+    o[0] = (uint32_t)best;
+    o[1] = (uint32_t)(best >> 32);
+    o[2] = bsl;
+    o[3] = hmin;
+  }
+  __syncwarp();
 }
 
-struct Summary {
-  uint32_t k, id, sl;
-};
+// One lane: recompute the record of SM s from its stored keys and H.
+__device__ void rescan_sm_lane(const Pt &P, uint32_t s, uint32_t H) {
+  const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
+  uint64_t best = INF64;
+  uint32_t bsl = 0, hmin = INF;
+  for (uint32_t i = i0; i < i1; i++) {
+    const uint32_t *sl = P.slot(i);
+    const uint32_t k = sl[F_KEY], h = sl[F_HID];
+    if (k == INF) continue;
+    const bool hb = (h & HBM_BIT) != 0u;
+    const uint64_t val = pack(hb ? max(k, H) : k, h & ID_MASK);
+    if (hb) hmin = min(hmin, k);
+    if (val < best) { best = val; bsl = i; }
+  }
+  uint32_t *o = P.smrec(s);
+  o[0] = (uint32_t)best;
+  o[1] = (uint32_t)(best >> 32);
+  o[2] = bsl;
+  o[3] = hmin;
+}
 
-// The lane's minimum over the SMs it owns.
-__device__ __forceinline__ Summary lane_summary(const Pt &P, int lane) {
-  Summary b{INF, NONE, 0};
+// Lane's best (packed, slot) over the SMs it owns, computed by that lane.
+__device__ __forceinline__ uint64_t lane_best(const Pt &P, int lane, uint32_t &slot) {
+  uint64_t b = INF64;
+  slot = 0;
   for (uint32_t s = lane; s < P.L.NS; s += 32) {
-    const uint32_t *o = P.sp + P.L.o_sm + s * SM_WORDS;
-    if (lex_less(o[0], o[1], b.k, b.id)) b = Summary{o[0], o[1], o[2]};
-    if (lex_less(o[3], o[4], b.k, b.id)) b = Summary{o[3], o[4], o[5]};
+    const uint2 o = *reinterpret_cast<const uint2 *>(P.smrec(s));
+    const uint64_t v = pack(o.y, o.x);
+    if (v < b) { b = v; slot = P.smrec(s)[2]; }
   }
   return b;
+}
+
+// Warp-parallel: the best over the SMs owned by lane `owner`; the owner lane
+// stores it in (b, bsl).
+__device__ __forceinline__ void refresh_owner(const Pt &P, uint32_t owner, int lane, uint64_t &b, uint32_t &bsl) {
+  uint64_t best = INF64;
+  uint32_t slot = 0;
+  for (uint32_t base = owner; base < P.L.NS; base += 32 * 32) {
+    const uint32_t s = base + 32u * lane;
+    uint64_t val = INF64;
+    if (s < P.L.NS) {
+      const uint2 o = *reinterpret_cast<const uint2 *>(P.smrec(s));
+      val = pack(o.y, o.x);
+    }
+    uint32_t who;
+    const uint64_t m = warp_min64(val, who);
+    const uint32_t ws = __shfl_sync(FULL, s < P.L.NS ? P.smrec(s)[2] : 0u, who);
+    if (m < best) { best = m; slot = ws; }
+  }
+  if ((uint32_t)lane == owner) { b = best; bsl = slot; }
 }
 
 // Slot i takes node v as its head (v == NONE: stream exhausted); adj_cnt /
@@ -314,21 +349,21 @@ __device__ __forceinline__ Summary lane_summary(const Pt &P, int lane) {
 // same values.
 __device__ __forceinline__ void set_head(const Pt &P, uint32_t i, uint32_t v, uint4 r, uint4 q, uint2 c,
                                          uint32_t adj_cnt, uint32_t adj_rdy) {
-  uint32_t *sp = P.sp;
+  uint32_t *sl = P.slot(i);
   if (v == NONE) {
-    sp[P.L.o_hid + i] = NONE;
-    sp[P.L.o_key + i] = INF;
-    sp[P.L.o_meta + i] = RC_NONE;
+    sl[F_HID] = NONE;
+    sl[F_KEY] = INF;
+    sl[F_META] = RC_NONE;
     return;
   }
   const uint32_t type = r.w & 15u;
   const uint32_t pend = (r.w >> 4) - c.x - adj_cnt;
   const uint32_t deg = min(q.w - q.z, DEG_BIG);
-  sp[P.L.o_hid + i] = v | (type_hbm(type) ? HBM_BIT : 0u);
-  sp[P.L.o_rdy + i] = max(c.y, adj_rdy);
-  sp[P.L.o_meta + i] = type_class(type) | (deg << 3) | (pend << 8);
-  sp[P.L.o_nxt + i] = r.z;
-  sp[P.L.o_sb + i] = q.z;
+  sl[F_HID] = v | (((TYPE_HBM >> type) & 1u) ? HBM_BIT : 0u);
+  sl[F_RDY] = max(c.y, adj_rdy);
+  sl[F_META] = ((TYPE_CLASS >> (4 * type)) & 15u) | (deg << 3) | (pend << 8);
+  sl[F_NXT] = r.z;
+  sl[F_SB] = q.z;
 }
 
 struct Clock {
@@ -340,17 +375,17 @@ struct Clock {
 };
 
 // Retire finished CTAs and launch as many CTAs as fit at cycle t (Section 5.1
-// TB scheduler; kernel-boundary gate).  Returns false on step-limit.  The
-// caller's lane summary `b` is refreshed when the lane owns a touched SM.
-__device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_row, int lane, Summary &b) {
-  uint32_t *sp = P.sp;
+// TB scheduler; kernel-boundary gate).  Returns false on step-limit.
+__device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_row, int lane, uint64_t &b,
+                            uint32_t &bsl) {
   const uint32_t t = C.t;
   for (;;) {
     uint32_t nr = INF;
     for (uint32_t j = lane; j < P.L.Scta; j += 32) {
-      if (sp[P.L.o_cid + j] != NONE && sp[P.L.o_crem + j] == 0u) {
-        if (sp[P.L.o_cend + j] <= t) sp[P.L.o_cid + j] = NONE;
-        else nr = min(nr, sp[P.L.o_cend + j]);
+      uint32_t *cr = P.cta(j);
+      if (cr[C_ID] != NONE && cr[C_REM] == 0u) {
+        if (cr[C_END] <= t) cr[C_ID] = NONE;
+        else nr = min(nr, cr[C_END]);
       }
     }
     C.next_ret = __reduce_min_sync(FULL, nr);
@@ -360,8 +395,9 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
     bool blocked = false;
     uint32_t freeslot = NONE;
     for (uint32_t j = lane; j < P.L.Scta; j += 32) {
-      if (sp[P.L.o_cid + j] != NONE) {
-        if (sp[P.L.o_ckern + j] < kc) blocked = true;
+      const uint32_t *cr = P.cta(j);
+      if (cr[C_ID] != NONE) {
+        if (cr[C_KERN] < kc) blocked = true;
       } else {
         freeslot = min(freeslot, j);
       }
@@ -373,10 +409,11 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
     const uint32_t c = C.next_cta;
     const uint32_t cnt = g.cta_cnt[c];
     if (lane == 0) {
-      sp[P.L.o_cid + freeslot] = c;
-      sp[P.L.o_crem + freeslot] = cnt;
-      sp[P.L.o_cend + freeslot] = 0u;
-      sp[P.L.o_ckern + freeslot] = kc;
+      uint32_t *cr = P.cta(freeslot);
+      cr[C_ID] = c;
+      cr[C_REM] = cnt;
+      cr[C_END] = 0u;
+      cr[C_KERN] = kc;
       if (cta_sm_row) cta_sm_row[c - P.c0] = (int32_t)(freeslot / P.cps);
       __threadfence();  // lane 0's earlier counter releases before the heads are read below
     }
@@ -393,15 +430,11 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
         cc = ld_counters(P.scr + (v - P.n0));
       }
       set_head(P, i, v, r, q, cc, 0u, 0u);
-      sp[P.L.o_key + i] = slot_key(P, i, t);
     }
     __syncwarp();
     const uint32_t s = freeslot / P.cps;
-    if ((uint32_t)lane == (s & 31u)) {
-      sm_summary(P, s, C.H);
-      b = lane_summary(P, lane);
-    }
-    __syncwarp();
+    refresh_sm(P, s, t, C.H, true, lane);
+    refresh_owner(P, s & 31u, lane, b, bsl);
     C.next_cta++;
   }
 }
@@ -452,25 +485,38 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     P.scr = scratch + (size_t)gw * ((g.row_nodes + 1u) & ~1u);
     int32_t *cta_sm_row = (flags & GTS_WANT_CTA_SM) ? d_cta_sm + (size_t)q * g.row_ctas : nullptr;
 
-    // ---- clear state
+    // ---- per-point constants and cleared state
     if (lane < (int)RC_N) {
       uint32_t off = 0;
       for (int r = 0; r < lane; r++) off += (uint32_t)prm[GTS_P_CAP_TENSOR + r];
       sp[O_CAP + lane] = (uint32_t)prm[GTS_P_CAP_TENSOR + lane];
       sp[O_OFF + lane] = off;
-      // the five rates sit at parameter indices 2, 4, 6, 8, 10 (HBM, TMA, SMEM, MMA, ALU)
       *reinterpret_cast<uint64_t *>(sp + O_MAG + 2 * lane) = div_const((uint32_t)prm[GTS_P_HBM_BPC + 2 * lane]);
     }
+    if (lane < 8) {  // base latency per type: LOAD, SMEM, MMA, EW, STORE, BAR, NOP
+      uint32_t bl = 0;
+      switch (lane) {
+        case GTS_LOAD: bl = (uint32_t)prm[GTS_P_TMA_LAT] + (uint32_t)prm[GTS_P_DRAM_LAT]; break;
+        case GTS_SMEM: bl = (uint32_t)prm[GTS_P_SMEM_LAT]; break;
+        case GTS_MMA: bl = (uint32_t)prm[GTS_P_MMA_LAT]; break;
+        case GTS_EW: bl = (uint32_t)prm[GTS_P_ALU_LAT]; break;
+        case GTS_STORE: bl = (uint32_t)prm[GTS_P_TMA_LAT]; break;
+        case GTS_BAR: bl = (uint32_t)prm[GTS_P_BAR_LAT]; break;
+        default: break;
+      }
+      sp[O_BASE + lane] = bl;
+    }
     for (uint32_t i = lane; i < P.L.S; i += 32) {
-      sp[P.L.o_hid + i] = NONE;
-      sp[P.L.o_key + i] = INF;
-      sp[P.L.o_meta + i] = RC_NONE;
+      uint32_t *sl = P.slot(i);
+      sl[F_HID] = NONE;
+      sl[F_KEY] = INF;
+      sl[F_META] = RC_NONE;
     }
     for (uint32_t s = lane; s < P.L.NS; s += 32) {
-      uint32_t *o = sp + P.L.o_sm + s * SM_WORDS;
-      o[0] = INF; o[1] = NONE; o[2] = 0; o[3] = INF; o[4] = NONE; o[5] = 0;
+      uint32_t *o = P.smrec(s);
+      o[0] = NONE; o[1] = INF; o[2] = 0; o[3] = INF;
     }
-    for (uint32_t j = lane; j < P.L.Scta; j += 32) sp[P.L.o_cid + j] = NONE;
+    for (uint32_t j = lane; j < P.L.Scta; j += 32) P.cta(j)[C_ID] = NONE;
     for (uint32_t k = lane; k < P.L.NS * P.L.SC; k += 32) sp[P.L.o_sv + k] = 0u;
     for (uint32_t k = lane; k < P.L.cap_hbm; k += 32) sp[P.L.o_hs + k] = 0u;
     {
@@ -494,32 +540,38 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     uint32_t issued = 0;
     int32_t mk = 0;
     uint64_t digest = 0;
-    Summary b{INF, NONE, 0};
-    if (!launch_ctas(g, P, C, cta_sm_row, lane, b)) status = GTS_ERR_STEP_LIMIT;
+    uint64_t b = INF64;  // this lane's best (effective cycle << 32 | id) over its SMs
+    uint32_t bsl = 0;    // ... and its slot
+    if (!launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
 
     while (status == GTS_OK && issued < nG) {
-      // ---- next event: lexicographic min of (effective cycle, node id) over all heads
-      const uint32_t E = __reduce_min_sync(FULL, b.k);
-      const uint32_t v = __reduce_min_sync(FULL, b.k == E ? b.id : NONE);
+      // ---- next event: minimum of (effective cycle, node id) over all heads
+      uint32_t owner;
+      const uint64_t m = warp_min64(b, owner);
+      const uint32_t E = (uint32_t)(m >> 32);
       if (E > C.t) {
         const uint32_t tn = min(E, C.next_ret);
         if (tn == INF) { status = GTS_ERR_DEADLOCK; break; }
         if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
         C.t = tn;
-        if (C.next_ret <= C.t && !launch_ctas(g, P, C, cta_sm_row, lane, b)) { status = GTS_ERR_STEP_LIMIT; break; }
+        if (C.next_ret <= C.t && !launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) {
+          status = GTS_ERR_STEP_LIMIT;
+          break;
+        }
         continue;
       }
       // ---- issue v, the lowest-id issuable head, at cycle t (all lanes, same values)
       if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
-      const uint32_t owner = __ffs(__ballot_sync(FULL, b.k == E && b.id == v)) - 1;
-      const uint32_t i = __shfl_sync(FULL, b.sl, owner);
+      const uint32_t v = (uint32_t)m;
+      const uint32_t i = __shfl_sync(FULL, bsl, owner);
       const uint32_t t = C.t;
       const uint32_t cs = i / P.W;
       const uint32_t sm = cs / P.cps;
-      const uint32_t hidv = sp[P.L.o_hid + i];
-      const uint32_t meta = sp[P.L.o_meta + i];
-      const uint32_t nx = sp[P.L.o_nxt + i];
-      const uint32_t sb = sp[P.L.o_sb + i];
+      uint32_t *sl = P.slot(i);
+      const uint2 s01 = *reinterpret_cast<const uint2 *>(sl + F_HID);
+      const uint2 s23 = *reinterpret_cast<const uint2 *>(sl + F_RDY);
+      const uint2 s45 = *reinterpret_cast<const uint2 *>(sl + F_NXT);
+      const uint32_t hidv = s01.x, meta = s23.y, nx = s45.x, sb = s45.y;
       const uint32_t cls = meta & 7u;
       // one round of independent loads: the issued node's record, the next
       // head's record, range and counters, and the successor entries
@@ -535,15 +587,14 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       if (deg == DEG_BIG) deg = g.rng[v].w - sb;
       uint2 ew = make_uint2(NONE, 0);
       if ((uint32_t)lane < deg) ew = g.succ[sb + lane];
-      cn.x = __shfl_sync(FULL, cn.x, 0);
-      cn.y = __shfl_sync(FULL, cn.y, 0);
       uint32_t occ, hocc;
       uint64_t lat;
       node_cost(sp, rv.w & 15u, rv.x, rv.y, occ, hocc, lat);
       const uint64_t f64 = (uint64_t)t + lat;
       if (f64 > 0x7FFFFFFFull) { status = GTS_ERR_OVERFLOW; break; }
       const uint32_t f = (uint32_t)f64;
-      __syncwarp();
+      cn.x = __shfl_sync(FULL, cn.x, 0);
+      cn.y = __shfl_sync(FULL, cn.y, 0);
       // take one free server of the node's class on its SM (lane k tests server k)
       if (cls != RC_NONE) {
         uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + sp[O_OFF + cls];
@@ -571,16 +622,18 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         }
         if (want_digest) digest += mix64(((uint64_t)(v - P.n0) << 32 | t) ^ ((uint64_t)f * 0x9E3779B97F4A7C15ull));
       }
-      const uint32_t rem = sp[P.L.o_crem + cs] - 1u;
-      const uint32_t cend = max(sp[P.L.o_cend + cs], f);
-      const uint32_t myc = sp[P.L.o_cid + cs];
+      uint32_t *cr = P.cta(cs);
+      const uint32_t rem = cr[C_REM] - 1u;
+      const uint32_t cend = max(cr[C_END], f);
+      const uint32_t myc = cr[C_ID];
       __syncwarp();
-      sp[P.L.o_crem + cs] = rem;
-      sp[P.L.o_cend + cs] = cend;
+      cr[C_REM] = rem;
+      cr[C_END] = cend;
       mk = max(mk, (int32_t)f);
       issued++;
       // ---- release successors, in edge order
       uint32_t adj_cnt = 0, adj_rdy = 0;
+      bool cross_touch = false;
       for (uint32_t base = 0; base < deg; base += 32) {
         if (base) ew = (base + lane < deg) ? g.succ[sb + base + lane] : make_uint2(NONE, 0);
         const uint32_t cnt = min(32u, deg - base);
@@ -599,17 +652,18 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
             tcs = cs;
           } else {
             for (uint32_t jj = 0; jj < P.L.Scta; jj++)
-              if (sp[P.L.o_cid + jj] == wc) { tcs = jj; break; }
+              if (P.cta(jj)[C_ID] == wc) { tcs = jj; break; }
           }
-          const uint32_t js = tcs * P.W + ((y >> 1) & 127u);
-          const bool head = tcs != NONE && (sp[P.L.o_hid + js] & ID_MASK) == w;
+          uint32_t *ts = P.slot(tcs * P.W + ((y >> 1) & 127u));
+          const bool head = tcs != NONE && (ts[F_HID] & ID_MASK) == w;
           if (head) {
-            const uint32_t m2 = sp[P.L.o_meta + js] - 256u;
-            const uint32_t r2 = max(sp[P.L.o_rdy + js], rel);
+            const uint32_t m2 = ts[F_META] - 256u;
+            const uint32_t r2 = max(ts[F_RDY], rel);
             __syncwarp();
-            sp[P.L.o_meta + js] = m2;
-            sp[P.L.o_rdy + js] = r2;
+            ts[F_META] = m2;
+            ts[F_RDY] = r2;
             __syncwarp();
+            cross_touch |= tcs != cs;
           } else if (lane == 0) {
             uint2 *c = P.scr + (w - P.n0);
             atomicAdd(&c->x, 1u);
@@ -620,27 +674,32 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       set_head(P, i, nx, rn, qn, cn, adj_cnt, adj_rdy);
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
-      if (g.cross_cta) {
-        for (uint32_t k = lane; k < P.L.S; k += 32) sp[P.L.o_key + k] = slot_key(P, k, t);
+      if (cross_touch) {  // a release reached a head of another CTA: recompute everything
+        for (uint32_t k = lane; k < P.L.S; k += 32) P.slot(k)[F_KEY] = slot_key(P, k, t);
         __syncwarp();
-        for (uint32_t s = lane; s < P.L.NS; s += 32) sm_summary(P, s, C.H);
-        b = lane_summary(P, lane);
+        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane(P, s, C.H);
+        __syncwarp();
+        b = lane_best(P, lane, bsl);
       } else {
-        const uint32_t k0 = sm * P.L.per;
-        for (uint32_t k = k0 + lane; k < min(k0 + P.L.per, P.L.S); k += 32) sp[P.L.o_key + k] = slot_key(P, k, t);
-        __syncwarp();
+        refresh_sm(P, sm, t, C.H, true, lane);
         if (C.H != prevH) {
-          for (uint32_t s = lane; s < P.L.NS; s += 32) sm_summary(P, s, C.H);
-          b = lane_summary(P, lane);
-        } else if ((uint32_t)lane == (sm & 31u)) {
-          sm_summary(P, sm, C.H);
-          b = lane_summary(P, lane);
+          // SMs whose HBM heads H overtakes change their effective cycles
+          bool any = false;
+          for (uint32_t s = lane; s < P.L.NS; s += 32) {
+            if (s != sm && P.smrec(s)[3] < C.H) {
+              rescan_sm_lane(P, s, C.H);
+              any = true;
+            }
+          }
+          if (any || (uint32_t)lane == (sm & 31u)) b = lane_best(P, lane, bsl);
+        } else {
+          refresh_owner(P, sm & 31u, lane, b, bsl);
         }
       }
       __syncwarp();
       if (rem == 0u) {
         if (cend <= t) {
-          if (!launch_ctas(g, P, C, cta_sm_row, lane, b)) { status = GTS_ERR_STEP_LIMIT; break; }
+          if (!launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
         } else {
           C.next_ret = min(C.next_ret, cend);
         }
