@@ -31,7 +31,7 @@ if ROOT not in sys.path:
 METRIC = "simulated tile-graph nodes/sec"
 UNIT = "node-points/s"
 KERNEL_SRC = os.path.join(ROOT, "paper_2607_11262_gb300", "csrc", "gts.cu")
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_k_simulate.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_k_simulate.txt")
 
 
 def node_points_of(graph, params):
@@ -252,7 +252,7 @@ def main():
     traffic = None
     if os.path.exists(TRAFFIC_FILE):
         tf = json.load(open(TRAFFIC_FILE))
-        if tf.get("source_sha256_16") == source_hash() and tf.get("workload") == w.name:
+        if tf.get("source_sha256_16") == source_hash() and w.name in tf.get("applies_to", []):
             traffic = tf["bytes_per_node_point"] * node_points + tf.get("bytes_fixed", 0)
     cb = None
     if not args.no_cpu_baseline:

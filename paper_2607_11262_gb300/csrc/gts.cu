@@ -106,6 +106,7 @@ struct DevGraph {
   const uint32_t *node_off;    // [G+1]
   const uint32_t *cta_off;     // [G+1]
   uint32_t W, G, row_nodes, row_ctas, cross_cta;
+  uint32_t class_mask;  // bit r: some node uses per-SM class r (servers of unused classes are not kept)
 };
 
 // ----------------------------------------------------------------- per-point layout
@@ -148,7 +149,8 @@ __host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
 // Fills `L` for a valid row on a graph with CG CTAs; false if the point needs
 // more than one warp's shared-memory budget.  Servers per class are limited
 // to 32 (one lane each).
-__host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint32_t W, Layout &L) {
+__host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint32_t W, uint32_t class_mask,
+                                          Layout &L) {
   const uint64_t cps = (uint64_t)p[GTS_P_CTAS_PER_SM];
   uint64_t slots = (uint64_t)p[GTS_P_NUM_SMS] * cps;
   if (slots > CG) slots = CG;
@@ -160,6 +162,7 @@ __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint3
   uint64_t sc = 0;
   for (int r = 0; r < (int)RC_N; r++) {
     const uint64_t c = (uint64_t)p[GTS_P_CAP_TENSOR + r];
+    if (!((class_mask >> r) & 1u)) continue;
     if (c > 32) return false;
     sc += c;
   }
@@ -468,7 +471,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     P.c1 = g.cta_off[gi + 1];
     const uint32_t CG = P.c1 - P.c0;
     if (status == GTS_OK) {
-      if (!make_layout(prm, CG, P.W, P.L) || P.L.words > budget_words) status = GTS_ERR_UNSUPPORTED;
+      if (!make_layout(prm, CG, P.W, g.class_mask, P.L) || P.L.words > budget_words) status = GTS_ERR_UNSUPPORTED;
     }
     if (status != GTS_OK) {
       if (lane == 0) {
@@ -486,10 +489,11 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     int32_t *cta_sm_row = (flags & GTS_WANT_CTA_SM) ? d_cta_sm + (size_t)q * g.row_ctas : nullptr;
 
     // ---- per-point constants and cleared state
-    if (lane < (int)RC_N) {
+    if (lane < (int)RC_N) {  // servers are kept only for the classes the graph uses
       uint32_t off = 0;
-      for (int r = 0; r < lane; r++) off += (uint32_t)prm[GTS_P_CAP_TENSOR + r];
-      sp[O_CAP + lane] = (uint32_t)prm[GTS_P_CAP_TENSOR + lane];
+      for (int r = 0; r < lane; r++)
+        if ((g.class_mask >> r) & 1u) off += (uint32_t)prm[GTS_P_CAP_TENSOR + r];
+      sp[O_CAP + lane] = ((g.class_mask >> lane) & 1u) ? (uint32_t)prm[GTS_P_CAP_TENSOR + lane] : 0u;
       sp[O_OFF + lane] = off;
       *reinterpret_cast<uint64_t *>(sp + O_MAG + 2 * lane) = div_const((uint32_t)prm[GTS_P_HBM_BPC + 2 * lane]);
     }
@@ -827,7 +831,7 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
     if (noff[k + 1] < noff[k] || coff[k + 1] < coff[k])
       return fail(GTS_ERR_INVALID_GRAPH, "graph offsets decrease at graph " + std::to_string(k));
   if (row_ptr[0] != 0 || row_ptr[n] != m) return fail(GTS_ERR_INVALID_GRAPH, "row_ptr[0] != 0 or row_ptr[n] != n_edges");
-  uint32_t row_nodes = 0, row_ctas = 0, cross = 0;
+  uint32_t row_nodes = 0, row_ctas = 0, cross = 0, class_mask = 0;
   for (uint64_t k = 0; k < G; k++) {
     const uint32_t n0 = noff[k], n1 = noff[k + 1], c0 = coff[k], c1 = coff[k + 1];
     row_nodes = std::max(row_nodes, n1 - n0);
@@ -835,6 +839,8 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
     for (uint32_t v = n0; v < n1; v++) {
       if (row_ptr[v + 1] < row_ptr[v]) return fail(GTS_ERR_INVALID_GRAPH, "row_ptr decreases at node " + std::to_string(v));
       if (ty[v] > GTS_NOP) return fail(GTS_ERR_INVALID_GRAPH, "bad type at node " + std::to_string(v));
+      const uint32_t cls_v = (TYPE_CLASS >> (4 * ty[v])) & 15u;
+      if (cls_v < RC_N) class_mask |= 1u << cls_v;
       if (wp[v] >= W) return fail(GTS_ERR_INVALID_GRAPH, "warp >= warps_per_cta at node " + std::to_string(v));
       if (cta[v] < c0 || cta[v] >= c1) return fail(GTS_ERR_INVALID_GRAPH, "cta outside its graph at node " + std::to_string(v));
       for (uint32_t x = row_ptr[v]; x < row_ptr[v + 1]; x++) {
@@ -904,6 +910,7 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   dg.row_nodes = row_nodes;
   dg.row_ctas = row_ctas;
   dg.cross_cta = cross;
+  dg.class_mask = class_mask;
   *out = g;
   return GTS_OK;
 }
@@ -934,7 +941,7 @@ gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_p
     if (check_row(row, g->G) != GTS_OK) continue;
     const uint32_t gi = (uint32_t)row[GTS_P_GRAPH_INDEX];
     Layout L;
-    if (make_layout(row, g->cta_off[gi + 1] - g->cta_off[gi], g->W, L)) P->words[p] = L.words;
+    if (make_layout(row, g->cta_off[gi + 1] - g->cta_off[gi], g->W, g->dg.class_mask, L)) P->words[p] = L.words;
   }
   *out = P;
   return GTS_OK;
