@@ -210,6 +210,35 @@ gts_status gts_read_results(gts_results *results, int32_t *h_makespan, int32_t *
                             uint64_t *h_digest, uint32_t n_points);
 gts_status gts_results_destroy(gts_results *results);
 
+/*
+ * No-allocation variant of gts_simulate_batch.  The paper has no counterpart:
+ * it is an interface for callers that cannot allocate device memory at the
+ * point of the call -- code running inside a CUDA graph being captured, under
+ * an allocator that must not grow, or in a host environment that owns every
+ * allocation itself.  Instead of caller scratch it uses one fixed array of
+ * GTS_STATIC_SCRATCH_BYTES that lives in the library's own device memory: every
+ * GPU that loads the library holds it until the process exits.  The caller
+ * still passes every input and output.
+ *  - The first call on a device looks up that array's address for the current
+ *    device (cudaGetSymbolAddress); make that first call before any stream
+ *    capture.  No call allocates or frees device memory.
+ *  - The graph set's largest graph must have at most GTS_STATIC_SCRATCH_BYTES/8
+ *    nodes, else GTS_ERR_NOMEM; fewer design points then run at a time than
+ *    with a large caller scratch (one per 8 bytes x nodes of the array).
+ *  - All calls share the array and the kernel clears each design point's part
+ *    before use, so nothing carries over between calls; calls that overlap on
+ *    the GPU (other streams, other threads) race on it and must be ordered by
+ *    the caller.
+ *  - No results handle is returned: read d_makespan / d_status directly.
+ * Errors: as gts_simulate_batch, plus NOMEM for a graph too large.
+ */
+#define GTS_STATIC_SCRATCH_BYTES (32u << 20)
+gts_status gts_simulate_batch_noalloc(gts_graph *graph, gts_params *params,
+                                      uint32_t first_point, uint32_t n_points, uint32_t flags,
+                                      int32_t *d_start, int32_t *d_finish,
+                                      int32_t *d_makespan, int32_t *d_status,
+                                      uint64_t *d_digest, int32_t *d_cta_sm, void *stream);
+
 /* Message for the calling thread's last non-OK host-side status ("" if none). */
 const char *gts_last_error(void);
 

@@ -51,6 +51,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstdint>
 #include <cstring>
 #include <new>
@@ -84,15 +85,28 @@ static_assert(GTS_P_TMA_BPC == GTS_P_HBM_BPC + 2 && GTS_P_SMEM_BPC == GTS_P_HBM_
                   GTS_P_MMA_FMA_PC == GTS_P_HBM_BPC + 6 && GTS_P_ALU_OPS_PC == GTS_P_HBM_BPC + 8,
               "rate k of the division-constant table sits at parameter index GTS_P_HBM_BPC + 2k");
 
-thread_local std::string g_err;
+thread_local char g_err[512];
 
-gts_status fail(gts_status s, const std::string &msg) {
-  g_err = msg;
+gts_status fail(gts_status s, const char *msg) {
+  size_t k = 0;
+  for (; msg[k] && k + 1 < sizeof(g_err); k++) g_err[k] = msg[k];
+  g_err[k] = 0;
   return s;
 }
 
+gts_status fail(gts_status s, const std::string &msg) { return fail(s, msg.c_str()); }
+
+void clear_error() { g_err[0] = 0; }
+
 gts_status cuda_fail(cudaError_t e, const char *what) {
-  return fail(GTS_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+  char buf[256];
+  size_t k = 0;
+  for (const char *p = what; *p && k < 200; p++) buf[k++] = *p;
+  buf[k++] = ':';
+  buf[k++] = ' ';
+  for (const char *p = cudaGetErrorString(e); *p && k + 1 < sizeof(buf); p++) buf[k++] = *p;
+  buf[k] = 0;
+  return fail(GTS_ERR_CUDA, (const char *)buf);
 }
 
 // ----------------------------------------------------------------- device graph
@@ -771,7 +785,7 @@ struct gts_results {
 
 extern "C" {
 
-const char *gts_last_error(void) { return g_err.c_str(); }
+const char *gts_last_error(void) { return g_err; }
 
 size_t gts_graph_workspace_bytes(uint32_t n_nodes, uint32_t n_edges, uint32_t n_ctas, uint32_t warps_per_cta,
                                  uint32_t n_graphs) {
@@ -784,7 +798,7 @@ uint32_t gts_row_nodes(const gts_graph *g) { return g ? g->dg.row_nodes : 0u; }
 uint32_t gts_row_ctas(const gts_graph *g) { return g ? g->dg.row_ctas : 0u; }
 
 gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **out) {
-  g_err.clear();
+  clear_error();
   if (!d || !out) return fail(GTS_ERR_INVALID_ARG, "null desc or out");
   *out = nullptr;
   const uint64_t n = d->n_nodes, m = d->n_edges, C = d->n_ctas, W = d->warps_per_cta, G = d->n_graphs;
@@ -922,7 +936,7 @@ gts_status gts_graph_destroy(gts_graph *g) {
 
 gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_points, void *stream,
                              gts_params **out) {
-  g_err.clear();
+  clear_error();
   if (!g || !out || (n_points && !d_params)) return fail(GTS_ERR_INVALID_ARG, "null graph, params or out");
   *out = nullptr;
   std::vector<int32_t> h;
@@ -1015,7 +1029,7 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
                               int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status,
                               uint64_t *d_digest, int32_t *d_cta_sm, void *d_scratch, size_t scratch_bytes,
                               void *stream, gts_results **out) {
-  g_err.clear();
+  clear_error();
   if (out) *out = nullptr;
   if (!g || !P || P->graph != g) return fail(GTS_ERR_INVALID_ARG, "null or mismatched graph / params");
   if (flags & ~(GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM)) return fail(GTS_ERR_INVALID_ARG, "unknown flag");
@@ -1054,7 +1068,7 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
 
 gts_status gts_read_results(gts_results *r, int32_t *h_makespan, int32_t *h_status, uint64_t *h_digest,
                             uint32_t n_points) {
-  g_err.clear();
+  clear_error();
   if (!r) return fail(GTS_ERR_INVALID_ARG, "null results");
   if (n_points > r->n_points) return fail(GTS_ERR_INVALID_ARG, "n_points exceeds the batch");
   if (h_digest && !r->d_digest) return fail(GTS_ERR_INVALID_ARG, "batch ran without WANT_DIGEST");
@@ -1074,6 +1088,58 @@ gts_status gts_read_results(gts_results *r, int32_t *h_makespan, int32_t *h_stat
 gts_status gts_results_destroy(gts_results *r) {
   delete r;
   return GTS_OK;
+}
+
+}  // extern "C"
+
+// ----------------------------------------------------------------- no-allocation entry point
+// Scratch for gts_simulate_batch_noalloc: a fixed array in the library's own
+// device memory, created when the module loads on a device and held until the
+// process exits.  In host code the symbol is only a handle; its device address
+// comes from cudaGetSymbolAddress, resolved once per device.
+static __device__ __align__(256) uint2 g_static_scratch[GTS_STATIC_SCRATCH_BYTES / sizeof(uint2)];
+
+namespace {
+constexpr int MAX_DEVICES = 64;
+void *g_static_ptr[MAX_DEVICES];
+std::atomic<int> g_static_lock{0};
+
+// Address of this device's static scratch (set-up on the first call per device).
+gts_status static_scratch(void **out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "simulate_noalloc: current device");
+  if (dev < 0 || dev >= MAX_DEVICES) return fail(GTS_ERR_UNSUPPORTED, "simulate_noalloc: device ordinal above 63");
+  while (g_static_lock.exchange(1, std::memory_order_acquire)) {
+  }
+  gts_status st = GTS_OK;
+  if (!g_static_ptr[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess) st = cuda_fail(e, "simulate_noalloc: static scratch address");
+    else g_static_ptr[dev] = p;
+  }
+  *out = g_static_ptr[dev];
+  g_static_lock.store(0, std::memory_order_release);
+  return st;
+}
+}  // namespace
+
+extern "C" {
+
+gts_status gts_simulate_batch_noalloc(gts_graph *g, gts_params *P, uint32_t first_point, uint32_t n_points,
+                                      uint32_t flags, int32_t *d_start, int32_t *d_finish, int32_t *d_makespan,
+                                      int32_t *d_status, uint64_t *d_digest, int32_t *d_cta_sm, void *stream) {
+  clear_error();
+  if (!g) return fail(GTS_ERR_INVALID_ARG, "null graph");
+  if (scratch_row_bytes(g) > GTS_STATIC_SCRATCH_BYTES)
+    return fail(GTS_ERR_NOMEM, "simulate_noalloc: a graph of the set has more nodes than the static scratch holds "
+                               "(GTS_STATIC_SCRATCH_BYTES / 8)");
+  void *scr = nullptr;
+  gts_status st = static_scratch(&scr);
+  if (st != GTS_OK) return st;
+  return gts_simulate_batch(g, P, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status, d_digest,
+                            d_cta_sm, scr, GTS_STATIC_SCRATCH_BYTES, stream, nullptr);
 }
 
 }  // extern "C"

@@ -33,9 +33,11 @@ GTS_FULL_TRACE = 1
 GTS_WANT_DIGEST = 2
 GTS_WANT_CTA_SM = 4
 
+GTS_STATIC_SCRATCH_BYTES = 32 << 20
+
 EXPORTS = ("gts_graph_workspace_bytes", "gts_graph_create", "gts_graph_destroy", "gts_params_upload",
            "gts_params_destroy", "gts_row_nodes", "gts_row_ctas", "gts_scratch_bytes", "gts_simulate_batch",
-           "gts_read_results", "gts_results_destroy", "gts_last_error")
+           "gts_read_results", "gts_results_destroy", "gts_simulate_batch_noalloc", "gts_last_error")
 
 
 class GtsError(RuntimeError):
@@ -89,6 +91,8 @@ def load():
     lib.gts_read_results.restype = i32
     lib.gts_results_destroy.argtypes = [vp]
     lib.gts_results_destroy.restype = i32
+    lib.gts_simulate_batch_noalloc.argtypes = [vp, vp, u32, u32, u32, vp, vp, vp, vp, vp, vp, vp]
+    lib.gts_simulate_batch_noalloc.restype = i32
     lib.gts_last_error.argtypes = []
     lib.gts_last_error.restype = ctypes.c_char_p
     _lib = lib
@@ -152,6 +156,14 @@ def gts_read_results(results, h_makespan, h_status, h_digest, n_points):
 
 def gts_results_destroy(results):
     _check(load().gts_results_destroy(results))
+
+
+def gts_simulate_batch_noalloc(graph, params, first_point, n_points, flags, d_start, d_finish, d_makespan,
+                               d_status, d_digest, d_cta_sm, stream=0):
+    """gts_simulate_batch without caller scratch: libgts uses its own fixed
+    device array (GTS_STATIC_SCRATCH_BYTES) and allocates nothing."""
+    _check(load().gts_simulate_batch_noalloc(graph, params, first_point, n_points, flags, d_start, d_finish,
+                                             d_makespan, d_status, d_digest, d_cta_sm, stream))
 
 
 def gts_last_error():

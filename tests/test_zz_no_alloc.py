@@ -1,0 +1,101 @@
+"""gts_simulate_batch_noalloc -- the entry point for callers that cannot
+allocate device memory when they call (inside stream capture, under a fixed
+allocator, or where the host owns every allocation) -- gives the same results
+as gts_simulate_batch with caller scratch, call after call.
+
+This file is collected last on purpose: it shares the library's static scratch
+with nothing else and must pass alone in a fresh process or after the rest.
+"""
+import numpy as np
+import pytest
+
+from paper_2607_11262_gb300 import workloads as W
+from tests import tinygraphs as TG
+
+pytestmark = pytest.mark.gpu
+
+FLAGS = 1 | 2 | 4  # full trace, digest, CTA placement
+
+
+@pytest.fixture(scope="module")
+def gts_mod():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2607_11262_gb300 import gts
+    gts.load()
+    return gts
+
+
+def _noalloc(gts, dg, dp, out, first=0, n=None):
+    import torch
+    n = dp.n_points - first if n is None else n
+    p = lambda t: 0 if t is None else t.data_ptr()  # noqa: E731
+    gts.gts_simulate_batch_noalloc(dg.handle, dp.handle, first, n, FLAGS, p(out.start), p(out.finish),
+                                   p(out.makespan), p(out.status), p(out.digest), p(out.cta_sm),
+                                   torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    return {k: getattr(out, k).cpu().numpy().copy() for k in ("makespan", "status", "start", "finish", "digest",
+                                                               "cta_sm")}
+
+
+def _reference(gts, dg, dp):
+    import torch
+    out = gts.simulate(dg, dp, flags=FLAGS)
+    torch.cuda.synchronize()
+    return {k: getattr(out, k).cpu().numpy().copy() for k in ("makespan", "status", "start", "finish", "digest",
+                                                               "cta_sm")}
+
+
+def _same(a, b):
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k   # integer cycles: bit-exact
+
+
+@pytest.mark.parametrize("case", ["gemm512", "ws_small", "stacked_dags"])
+def test_noalloc_matches_caller_scratch_twice(gts_mod, case):
+    gts = gts_mod
+    if case == "gemm512":
+        w = W.workload("gemm512")
+        graph, params = w.graph, w.params
+    elif case == "ws_small":
+        w = W.workload("wsgemm_small", points=300)
+        graph, params = w.graph, w.params
+    else:
+        graph = W.stress_set(4, n_nodes=2500)
+        params = W.stress_params(4)
+    dg = gts.DeviceGraph(graph)
+    dp = gts.DeviceParams(dg, params)
+    ref = _reference(gts, dg, dp)
+    assert np.all(ref["status"] == 0)
+    out = gts.alloc_outputs(dg, dp.n_points, FLAGS)
+    first = _noalloc(gts, dg, dp, out)
+    _same(first, ref)
+    out.makespan.fill_(-7)
+    out.start.fill_(-7)
+    second = _noalloc(gts, dg, dp, out)  # the static array keeps the first call's contents
+    _same(second, ref)
+
+
+def test_noalloc_partial_range_and_too_large(gts_mod):
+    gts = gts_mod
+    w = W.workload("gemm512")
+    dg = gts.DeviceGraph(w.graph)
+    dp = gts.DeviceParams(dg, w.params)
+    ref = _reference(gts, dg, dp)
+    out = gts.alloc_outputs(dg, 20, FLAGS)
+    part = _noalloc(gts, dg, dp, out, first=10, n=20)
+    for k in part:
+        assert np.array_equal(part[k], ref[k][10:30]), k
+    # a graph with more nodes than the static array holds is refused
+    n = gts.GTS_STATIC_SCRATCH_BYTES // 8 + 2
+    big = W.from_edges("big", 1, np.full(n, W.NOP, np.uint8), np.zeros(n, np.uint16), np.zeros(n, np.uint32),
+                       np.zeros(n, np.uint32), np.zeros(n, np.uint32), np.zeros(1, np.uint32), [], [], [])
+    dgb = gts.DeviceGraph(big)
+    dpb = gts.DeviceParams(dgb, TG.unit_params()[None, :])
+    outb = gts.alloc_outputs(dgb, 1, 0)
+    with pytest.raises(gts.GtsError) as e:
+        gts.gts_simulate_batch_noalloc(dgb.handle, dpb.handle, 0, 1, 0, 0, 0, outb.makespan.data_ptr(),
+                                       outb.status.data_ptr(), 0, 0, 0)
+    assert e.value.status == gts.GTS_ERR_NOMEM
+    assert "static scratch" in gts.gts_last_error()
