@@ -102,6 +102,22 @@ class Clocks:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def reduce_max_over_ranks(value, device=None):
+    """Max of a per-rank float over the process group (identity without one)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(node_points_per_rank, world, ms_per_step):
+    """Whole-job throughput: every rank's node-points over the slowest rank's time."""
+    return node_points_per_rank * world / (ms_per_step / 1e3)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
@@ -133,9 +149,11 @@ def cpu_baseline(graph, params, seconds=15.0, procs=None):
     k = int(max(1, min(params.shape[0], procs * max(1, round(seconds / max(t_one, 1e-3))))))
     k = max(1, min(k, procs * 4))
     pts = list(range(k))
+    pool = oracle_run.PointPool(graph, min(procs, k))
     t0 = time.time()
-    res = oracle_run.simulate_points(graph, params, pts, processes=min(procs, k))
+    res = pool.run(params, pts)
     wall = time.time() - t0
+    pool.close()
     assert all(r.status == 0 for r in res.values())
     nodes = node_points_of(graph, params[pts])
     return {"value": nodes / wall, "unit": UNIT, "cores": min(procs, k), "kind": "oracle",
@@ -227,12 +245,9 @@ def main():
     total_ms = float(sum(step_ms))
     st = out.status.cpu().numpy()
     assert np.all(st == 0), f"non-OK statuses: {np.unique(st)}"
-    if ws > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = reduce_max_over_ranks(total_ms, device="cuda")
     ms_per_step = total_ms / args.steps
-    value = node_points * ws / (ms_per_step / 1e3)
+    value = whole_job_rate(node_points, ws, ms_per_step)
 
     # ---- e2e: host buffers through the C ABI, copies inside the timed region
     e2e = None

@@ -118,6 +118,30 @@ def _pool_run(args):
     return p, r
 
 
+def _pool_ready(_):
+    return os.getpid()
+
+
+class PointPool:
+    """A started pool of oracle worker processes holding one graph.
+
+    Start-up (spawning, shipping the graph, loading the library) happens in the
+    constructor, so ``run`` times only the simulation of the points."""
+
+    def __init__(self, graph, processes):
+        import multiprocessing as mp
+        self.processes = max(1, int(processes))
+        self.pool = mp.get_context("spawn").Pool(self.processes, initializer=_pool_init, initargs=(graph,))
+        self.pool.map(_pool_ready, range(self.processes * 2))
+
+    def run(self, params, points):
+        return dict(self.pool.imap_unordered(_pool_run, [(p, params[p]) for p in points]))
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+
+
 def simulate_points(graph, params, points, processes=None):
     """Oracle results for the listed points, computed in ``processes`` worker
     processes (spawned, so the pool is safe to start after CUDA init)."""
