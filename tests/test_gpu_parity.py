@@ -67,6 +67,18 @@ def test_random_small_graphs():
         _check_all(g, prms, res)
 
 
+def test_random_intra_cta_graphs():
+    rng = np.random.default_rng(22)
+    for i in range(80):
+        n = int(rng.integers(1, 70))
+        g = TG.random_graph(rng, n, W_=int(rng.integers(1, 6)), C=int(rng.integers(1, 7)),
+                            p_edge=float(rng.uniform(0.05, 0.4)), cta_major=True, kernels=bool(i % 2),
+                            intra_cta=True)
+        prms = np.stack([TG.small_params(rng, cps=1) for _ in range(4)]
+                        + [TG.small_params(rng, num_sms=4, cps=2) for _ in range(2)])
+        _check_all(g, prms, H.run_gpu(g, prms))
+
+
 def test_small_ws_gemm_many_tiles_ragged():
     # 5 persistent CTAs over 13 tiles (3,3,3,2,2), 6 k-steps, 4-stage ring
     per = [3, 3, 3, 2, 2]
@@ -90,6 +102,7 @@ def test_small_fa_and_decoder_shapes():
     ck = [0, 0, 1, 1, 1, 2, 2, 3, 3, 4]
     dec = W.assemble("dec", 4, tpls, np.array(ct), np.array(ck, np.uint32))
     p = W.sweep_params(7, 24, [(W.P_NUM_SMS, 1, 4), W.AX_HBM, W.AX_TMA_LAT, W.AX_MMA_RATE, W.AX_ALU_RATE], 1)
+    p[:4, W.P_CAP_HBM] = 2
     _check_all(dec, p, H.run_gpu(dec, p))
 
 

@@ -55,19 +55,22 @@ def make(n, edges, types, warps, ctas, W_, kernels=None, work=None, lat_extra=No
 
 
 def random_graph(rng, n, W_=None, C=None, p_edge=0.25, p_issue=0.3, max_work=6, cta_major=True,
-                 kernels=False, types=(0, 1, 2, 3, 4, 5, 6)):
-    """Random DAG over ids 0..n-1 (edges only go forward)."""
+                 kernels=False, types=(0, 1, 2, 3, 4, 5, 6), intra_cta=False):
+    """Random DAG over ids 0..n-1 (edges only go forward; with ``intra_cta``
+    only between nodes of the same CTA)."""
     W_ = W_ if W_ is not None else int(rng.integers(1, 4))
     C = C if C is not None else int(rng.integers(1, 4))
-    edges = []
-    for v in range(n):
-        for u in range(v):
-            if rng.random() < p_edge:
-                edges.append((u, v, int(rng.random() < p_issue)))
     if cta_major:
         ctas = sorted(int(x) for x in rng.integers(0, C, n))
     else:
         ctas = [int(x) for x in rng.integers(0, C, n)]
+    edges = []
+    for v in range(n):
+        for u in range(v):
+            if intra_cta and ctas[u] != ctas[v]:
+                continue
+            if rng.random() < p_edge:
+                edges.append((u, v, int(rng.random() < p_issue)))
     C_eff = max(ctas) + 1 if n else C
     C_eff = max(C_eff, C)
     warps = [int(x) for x in rng.integers(0, W_, n)]
