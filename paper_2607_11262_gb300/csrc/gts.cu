@@ -66,7 +66,7 @@ constexpr uint64_t INF64 = ~0ull;
 constexpr uint32_t HBM_BIT = 0x80000000u;  // on a slot's node id: node uses HBM
 constexpr uint32_t ID_MASK = 0x7FFFFFFFu;
 constexpr uint32_t FULL = 0xFFFFFFFFu;
-constexpr int MAX_WPB = 4;                  // warps (design points) per block
+constexpr int MAX_WPB = 4;                  // warps (design points) per block, at most
 constexpr uint32_t MAX_SMEM_BYTES = 227u * 1024u;
 constexpr uint32_t MAX_W = 128;
 constexpr uint32_t MAX_INDEG = (1u << 24) - 1;
@@ -128,17 +128,17 @@ struct DevGraph {
 // warp; CTA slot j lives on SM j / ctas_per_sm (SM-major, so the lowest free
 // slot is on the lowest SM with room).  Only min(num_sms*cps, C) CTA slots can
 // ever be occupied (a launch always takes the lowest free slot).
-constexpr uint32_t O_CAP = GTS_NPARAM;       // 5 words: servers per class
-constexpr uint32_t O_OFF = GTS_NPARAM + 5;   // 5 words: class offset inside an SM's servers
-constexpr uint32_t O_MAG = GTS_NPARAM + 10;  // 5 x 2 words: division constants of the rates
-constexpr uint32_t O_BASE = GTS_NPARAM + 20; // 8 words: base latency per node type
-constexpr uint32_t O_DYN = GTS_NPARAM + 28;  // first per-point array (16-byte aligned)
-// slot record (6 words): id|HBM, key, rdy, pending<<8 | deg<<3 | class, next, successor begin
-constexpr uint32_t F_HID = 0, F_KEY = 1, F_RDY = 2, F_META = 3, F_NXT = 4, F_SB = 5, SLOT_WORDS = 6;
+constexpr uint32_t O_MAG = GTS_NPARAM;       // 5 x 2 words: division constants of the rates (8-byte aligned)
+constexpr uint32_t O_BASE = GTS_NPARAM + 10; // 8 words: base latency per node type
+constexpr uint32_t O_DYN = GTS_NPARAM + 18;  // first per-point array
+static_assert(O_MAG % 2 == 0, "division constants are 8-byte words");
+// slot record (5 words): id|HBM, rdy, pending<<8 | deg<<3 | class, next, successor begin
+constexpr uint32_t F_HID = 0, F_RDY = 1, F_META = 2, F_NXT = 3, F_SB = 4, SLOT_WORDS = 5;
 // SM record (4 words): best id, best effective cycle, best slot, min key of its HBM heads
 constexpr uint32_t SM_WORDS = 4;
-// CTA slot record (4 words): CTA id, nodes not issued, max finish, kernel
-constexpr uint32_t C_ID = 0, C_REM = 1, C_END = 2, C_KERN = 3, CTA_WORDS = 4;
+static_assert(SM_WORDS % 2 == 0, "SM records are read as 8-byte pairs");
+// CTA slot record (3 words): CTA id, nodes not issued, max finish
+constexpr uint32_t C_ID = 0, C_REM = 1, C_END = 2, CTA_WORDS = 3;
 
 struct Layout {
   uint32_t S, Scta, NS, SC, cap_hbm, per;
@@ -185,6 +185,7 @@ __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint3
   L.cap_hbm = (uint32_t)p[GTS_P_CAP_HBM];
   uint64_t w = O_DYN;
   L.o_slot = (uint32_t)w; w += (uint64_t)L.S * SLOT_WORDS;
+  w = (w + 1) & ~(uint64_t)1;  // SM records are read as 8-byte pairs
   L.o_sm = (uint32_t)w; w += (uint64_t)L.NS * SM_WORDS;
   L.o_cta = (uint32_t)w; w += (uint64_t)L.Scta * CTA_WORDS;
   L.o_sv = (uint32_t)w; w += (uint64_t)L.NS * L.SC;
@@ -235,6 +236,10 @@ struct Pt {
   uint32_t W, cps, n0, c0, c1;
   int32_t *st, *fi;  // trace rows (graph-local index) or null
   uint2 *scr;        // scratch counters (graph-local index)
+  uint64_t offs;     // byte r: offset of class r's servers inside an SM's servers
+  uint32_t caps;     // 6 bits per class: servers of class r (0: class unused)
+  __device__ __forceinline__ uint32_t cls_off(uint32_t r) const { return (uint32_t)(offs >> (8 * r)) & 255u; }
+  __device__ __forceinline__ uint32_t cls_cap(uint32_t r) const { return (caps >> (6 * r)) & 63u; }
   __device__ __forceinline__ uint32_t *slot(uint32_t i) const { return sp + L.o_slot + i * SLOT_WORDS; }
   __device__ __forceinline__ uint32_t *smrec(uint32_t s) const { return sp + L.o_sm + s * SM_WORDS; }
   __device__ __forceinline__ uint32_t *cta(uint32_t j) const { return sp + L.o_cta + j * CTA_WORDS; }
@@ -261,8 +266,8 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
   const uint32_t cls = meta & 7u;
   if (cls != RC_NONE) {
     const uint32_t sm = i / P.L.per;
-    const uint32_t *sv = P.sp + P.L.o_sv + sm * P.L.SC + P.sp[O_OFF + cls];
-    const uint32_t cap = P.sp[O_CAP + cls];
+    const uint32_t *sv = P.sp + P.L.o_sv + sm * P.L.SC + P.cls_off(cls);
+    const uint32_t cap = P.cls_cap(cls);
     uint32_t a = sv[0];
     for (uint32_t q = 1; q < cap; q++) a = min(a, sv[q]);
     k = max(k, a);
@@ -270,9 +275,9 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
   return k;
 }
 
-// Warp-parallel: recompute (when `keys`) the keys of SM s's slots at cycle t
-// and its summary record.  All lanes call it.
-__device__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, bool keys, int lane) {
+// Warp-parallel: the keys of SM s's heads at cycle t and the SM's summary
+// record.  All lanes call it.
+__device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane) {
   const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
   uint64_t best = INF64;
   uint32_t bsl = 0, hmin = INF;
@@ -280,10 +285,8 @@ __device__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, bool
     const uint32_t i = base + lane;
     uint64_t val = INF64;
     if (i < i1) {
-      uint32_t *sl = P.slot(i);
-      const uint32_t k = keys ? slot_key(P, i, t) : sl[F_KEY];
-      if (keys) sl[F_KEY] = k;
-      const uint32_t h = sl[F_HID];
+      const uint32_t k = slot_key(P, i, t);
+      const uint32_t h = P.slot(i)[F_HID];
       if (k != INF) {
         const bool hb = (h & HBM_BIT) != 0u;
         val = pack(hb ? max(k, H) : k, h & ID_MASK);
@@ -308,15 +311,15 @@ __device__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, bool
   __syncwarp();
 }
 
-// One lane: recompute the record of SM s from its stored keys and H.
-__device__ void rescan_sm_lane(const Pt &P, uint32_t s, uint32_t H) {
+// One lane: recompute the record of SM s at cycle t and horizon H.
+__device__ __forceinline__ void rescan_sm_lane(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
   const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
   uint64_t best = INF64;
   uint32_t bsl = 0, hmin = INF;
   for (uint32_t i = i0; i < i1; i++) {
-    const uint32_t *sl = P.slot(i);
-    const uint32_t k = sl[F_KEY], h = sl[F_HID];
+    const uint32_t k = slot_key(P, i, t);
     if (k == INF) continue;
+    const uint32_t h = P.slot(i)[F_HID];
     const bool hb = (h & HBM_BIT) != 0u;
     const uint64_t val = pack(hb ? max(k, H) : k, h & ID_MASK);
     if (hb) hmin = min(hmin, k);
@@ -369,7 +372,6 @@ __device__ __forceinline__ void set_head(const Pt &P, uint32_t i, uint32_t v, ui
   uint32_t *sl = P.slot(i);
   if (v == NONE) {
     sl[F_HID] = NONE;
-    sl[F_KEY] = INF;
     sl[F_META] = RC_NONE;
     return;
   }
@@ -414,7 +416,7 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
     for (uint32_t j = lane; j < P.L.Scta; j += 32) {
       const uint32_t *cr = P.cta(j);
       if (cr[C_ID] != NONE) {
-        if (cr[C_KERN] < kc) blocked = true;
+        if (g.cta_kernel[cr[C_ID]] < kc) blocked = true;
       } else {
         freeslot = min(freeslot, j);
       }
@@ -430,7 +432,6 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
       cr[C_ID] = c;
       cr[C_REM] = cnt;
       cr[C_END] = 0u;
-      cr[C_KERN] = kc;
       if (cta_sm_row) cta_sm_row[c - P.c0] = (int32_t)(freeslot / P.cps);
       __threadfence();  // lane 0's earlier counter releases before the heads are read below
     }
@@ -450,13 +451,13 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
     }
     __syncwarp();
     const uint32_t s = freeslot / P.cps;
-    refresh_sm(P, s, t, C.H, true, lane);
+    refresh_sm(P, s, t, C.H, lane);
     refresh_owner(P, s & 31u, lane, b, bsl);
     C.next_cta++;
   }
 }
 
-__global__ void __launch_bounds__(MAX_WPB * 32)
+__global__ void __launch_bounds__(MAX_WPB * 32, 1)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
            int32_t *d_cta_sm, uint2 *scratch, uint32_t n_warps, uint32_t budget_words) {
@@ -503,12 +504,18 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     int32_t *cta_sm_row = (flags & GTS_WANT_CTA_SM) ? d_cta_sm + (size_t)q * g.row_ctas : nullptr;
 
     // ---- per-point constants and cleared state
-    if (lane < (int)RC_N) {  // servers are kept only for the classes the graph uses
+    {  // servers are kept only for the classes the graph uses (caps <= 32, offsets < 160)
       uint32_t off = 0;
-      for (int r = 0; r < lane; r++)
-        if ((g.class_mask >> r) & 1u) off += (uint32_t)prm[GTS_P_CAP_TENSOR + r];
-      sp[O_CAP + lane] = ((g.class_mask >> lane) & 1u) ? (uint32_t)prm[GTS_P_CAP_TENSOR + lane] : 0u;
-      sp[O_OFF + lane] = off;
+      P.offs = 0;
+      P.caps = 0;
+      for (uint32_t r = 0; r < RC_N; r++) {
+        const uint32_t c = ((g.class_mask >> r) & 1u) ? (uint32_t)prm[GTS_P_CAP_TENSOR + r] : 0u;
+        P.offs |= (uint64_t)off << (8 * r);
+        P.caps |= c << (6 * r);
+        off += c;
+      }
+    }
+    if (lane < (int)RC_N) {
       *reinterpret_cast<uint64_t *>(sp + O_MAG + 2 * lane) = div_const((uint32_t)prm[GTS_P_HBM_BPC + 2 * lane]);
     }
     if (lane < 8) {  // base latency per type: LOAD, SMEM, MMA, EW, STORE, BAR, NOP
@@ -527,7 +534,6 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     for (uint32_t i = lane; i < P.L.S; i += 32) {
       uint32_t *sl = P.slot(i);
       sl[F_HID] = NONE;
-      sl[F_KEY] = INF;
       sl[F_META] = RC_NONE;
     }
     for (uint32_t s = lane; s < P.L.NS; s += 32) {
@@ -585,11 +591,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       const uint32_t t = C.t;
       const uint32_t cs = i / P.W;
       const uint32_t sm = cs / P.cps;
-      uint32_t *sl = P.slot(i);
-      const uint2 s01 = *reinterpret_cast<const uint2 *>(sl + F_HID);
-      const uint2 s23 = *reinterpret_cast<const uint2 *>(sl + F_RDY);
-      const uint2 s45 = *reinterpret_cast<const uint2 *>(sl + F_NXT);
-      const uint32_t hidv = s01.x, meta = s23.y, nx = s45.x, sb = s45.y;
+      const uint32_t *sl = P.slot(i);
+      const uint32_t hidv = sl[F_HID], meta = sl[F_META], nx = sl[F_NXT], sb = sl[F_SB];
       const uint32_t cls = meta & 7u;
       // one round of independent loads: the issued node's record, the next
       // head's record, range and counters, and the successor entries
@@ -615,8 +618,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       cn.y = __shfl_sync(FULL, cn.y, 0);
       // take one free server of the node's class on its SM (lane k tests server k)
       if (cls != RC_NONE) {
-        uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + sp[O_OFF + cls];
-        const bool fr = (uint32_t)lane < sp[O_CAP + cls] && sv[lane] <= t;
+        uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + P.cls_off(cls);
+        const bool fr = (uint32_t)lane < P.cls_cap(cls) && sv[lane] <= t;
         const uint32_t bal = __ballot_sync(FULL, fr);
         if (lane == __ffs(bal) - 1) sv[lane] = t + occ;
       }
@@ -693,19 +696,17 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
       if (cross_touch) {  // a release reached a head of another CTA: recompute everything
-        for (uint32_t k = lane; k < P.L.S; k += 32) P.slot(k)[F_KEY] = slot_key(P, k, t);
-        __syncwarp();
-        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane(P, s, C.H);
+        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane(P, s, t, C.H);
         __syncwarp();
         b = lane_best(P, lane, bsl);
       } else {
-        refresh_sm(P, sm, t, C.H, true, lane);
+        refresh_sm(P, sm, t, C.H, lane);
         if (C.H != prevH) {
           // SMs whose HBM heads H overtakes change their effective cycles
           bool any = false;
           for (uint32_t s = lane; s < P.L.NS; s += 32) {
             if (s != sm && P.smrec(s)[3] < C.H) {
-              rescan_sm_lane(P, s, C.H);
+              rescan_sm_lane(P, s, t, C.H);
               any = true;
             }
           }
@@ -991,7 +992,7 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
   // warps per block: whichever keeps the most design points resident per SM
   uint32_t best_w = 0;
   pl.wpb = 1;
-  for (uint32_t wpb = MAX_WPB; wpb >= 1; wpb /= 2) {
+  for (uint32_t wpb = MAX_WPB; wpb >= 1; wpb--) {
     if (wpb * bytes > MAX_SMEM_BYTES) continue;
     int nb = 0;
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_simulate, (int)wpb * 32, wpb * bytes);
