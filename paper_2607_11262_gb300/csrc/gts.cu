@@ -578,11 +578,11 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         if (tn == INF) { status = GTS_ERR_DEADLOCK; break; }
         if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
         C.t = tn;
-        if (C.next_ret <= C.t && !launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) {
-          status = GTS_ERR_STEP_LIMIT;
-          break;
+        if (C.next_ret <= C.t) {  // a CTA retires first: launch, then choose again
+          if (!launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
+          continue;
         }
-        continue;
+        // otherwise the minimum just found is the first issue at the new cycle
       }
       // ---- issue v, the lowest-id issuable head, at cycle t (all lanes, same values)
       if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
