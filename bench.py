@@ -213,7 +213,7 @@ def main():
     P = int(w.params.shape[0])
     n = g.max_graph_nodes
     node_points = node_points_of(g, w.params)
-    flags = gts.GTS_FULL_TRACE | gts.GTS_WANT_DIGEST
+    flags = gts.GTS_FULL_TRACE
     stream = torch.cuda.Stream()
 
     with torch.cuda.stream(stream):

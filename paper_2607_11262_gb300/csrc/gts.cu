@@ -652,22 +652,18 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       cr[C_END] = cend;
       mk = max(mk, (int32_t)f);
       issued++;
-      // ---- release successors, in edge order
+      // ---- release successors, one per lane: into warp heads with shared-memory
+      // atomics; into scratch counters by lane 0 (which also reads them later)
       uint32_t adj_cnt = 0, adj_rdy = 0;
       bool cross_touch = false;
       for (uint32_t base = 0; base < deg; base += 32) {
         if (base) ew = (base + lane < deg) ? g.succ[sb + base + lane] : make_uint2(NONE, 0);
-        const uint32_t cnt = min(32u, deg - base);
-        for (uint32_t j = 0; j < cnt; j++) {
-          const uint32_t w = __shfl_sync(FULL, ew.x, j);
-          const uint32_t y = __shfl_sync(FULL, ew.y, j);
-          const uint32_t rel = (y & 1u) ? t : f;
-          if (w == nx) {  // the stream's next node becomes the head right below
-            adj_cnt++;
-            adj_rdy = max(adj_rdy, rel);
-            continue;
-          }
-          const uint32_t wc = y >> 8;
+        const bool mine = base + lane < deg;
+        const uint32_t rel = (ew.y & 1u) ? t : f;
+        const bool to_next = mine && ew.x == nx;  // the stream's next node becomes the head right below
+        bool to_head = false, cross = false;
+        if (mine && !to_next) {
+          const uint32_t wc = ew.y >> 8;
           uint32_t tcs = NONE;
           if (wc == myc) {
             tcs = cs;
@@ -675,23 +671,33 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
             for (uint32_t jj = 0; jj < P.L.Scta; jj++)
               if (P.cta(jj)[C_ID] == wc) { tcs = jj; break; }
           }
-          uint32_t *ts = P.slot(tcs * P.W + ((y >> 1) & 127u));
-          const bool head = tcs != NONE && (ts[F_HID] & ID_MASK) == w;
-          if (head) {
-            const uint32_t m2 = ts[F_META] - 256u;
-            const uint32_t r2 = max(ts[F_RDY], rel);
-            __syncwarp();
-            ts[F_META] = m2;
-            ts[F_RDY] = r2;
-            __syncwarp();
-            cross_touch |= tcs != cs;
-          } else if (lane == 0) {
+          if (tcs != NONE) {
+            uint32_t *ts = P.slot(tcs * P.W + ((ew.y >> 1) & 127u));
+            if ((ts[F_HID] & ID_MASK) == ew.x) {
+              atomicSub(&ts[F_META], 256u);
+              atomicMax(&ts[F_RDY], rel);
+              to_head = true;
+              cross = tcs != cs;
+            }
+          }
+        }
+        adj_cnt += __reduce_add_sync(FULL, to_next ? 1u : 0u);
+        adj_rdy = max(adj_rdy, __reduce_max_sync(FULL, to_next ? rel : 0u));
+        cross_touch |= __any_sync(FULL, cross);
+        uint32_t todo = __ballot_sync(FULL, mine && !to_next && !to_head);
+        while (todo) {
+          const int j = __ffs(todo) - 1;
+          todo &= todo - 1;
+          const uint32_t w = __shfl_sync(FULL, ew.x, j);
+          const uint32_t r = __shfl_sync(FULL, rel, j);
+          if (lane == 0) {
             uint2 *c = P.scr + (w - P.n0);
             atomicAdd(&c->x, 1u);
-            atomicMax(&c->y, rel);
+            atomicMax(&c->y, r);
           }
         }
       }
+      __syncwarp();
       set_head(P, i, nx, rn, qn, cn, adj_cnt, adj_rdy);
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
