@@ -126,7 +126,10 @@ def dist_env():
 def load_workload(name, rank, points):
     from paper_2607_11262_gb300 import workloads as W
     w = W.workload(name)
-    if rank > 0 and name != "stress":
+    if rank > 0 and name == "pipelines":
+        from paper_2607_11262_gb300 import pipelines
+        w.params = pipelines.study_params(w.graph.n_graphs, 64, seed=W.SEED0 + 6 + 100 * rank)
+    elif rank > 0 and name != "stress":
         # weak scaling: every rank gets its own design points of the same sweep
         axes = {"gemm512": [W.AX_SMS, W.AX_HBM, (W.P_MMA_LAT, 16, 64)],
                 "wsgemm8192": [W.AX_SMS, W.AX_HBM, W.AX_TMA_LAT, W.AX_MMA_RATE]}.get(

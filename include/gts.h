@@ -107,6 +107,21 @@ typedef int32_t gts_status;
 #define GTS_FULL_TRACE  1u  /* write d_start / d_finish [n_points][row_nodes] */
 #define GTS_WANT_DIGEST 2u  /* write d_digest[n_points] */
 #define GTS_WANT_CTA_SM 4u  /* write d_cta_sm [n_points][row_ctas] (-1: never launched) */
+#define GTS_WANT_BUSY   8u  /* write d_busy [n_points][GTS_BUSY_CLASSES] */
+
+/* Busy server-cycles per resource class (Section 5.2 throughput servers):
+ * d_busy[q*GTS_BUSY_CLASSES + r] = sum over the point's nodes v that use class
+ * r of occ_r(v), the cycles v holds one server of r.  Class r's utilisation
+ * over the run (Section 7.1 reports it for the tensor cores) is
+ * busy_r / (servers_r * makespan), with servers_r = cap_r * num_sms for the
+ * per-SM classes and cap_hbm for HBM. */
+#define GTS_BUSY_CLASSES 6
+#define GTS_BUSY_TENSOR  0
+#define GTS_BUSY_TMA     1
+#define GTS_BUSY_LSU     2
+#define GTS_BUSY_ALU     3
+#define GTS_BUSY_BAR     4
+#define GTS_BUSY_HBM     5
 
 typedef struct gts_graph gts_graph;
 typedef struct gts_params gts_params;
@@ -188,7 +203,8 @@ size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint3
  *   d_start[q*row_nodes + v], d_finish[...]         (GTS_FULL_TRACE; graph-local v)
  *   d_digest[q]                                     (GTS_WANT_DIGEST)
  *   d_cta_sm[q*row_ctas + c]                        (GTS_WANT_CTA_SM; graph-local c)
- * Start/finish/digest/cta_sm of a point whose status is not GTS_OK are
+ *   d_busy[q*GTS_BUSY_CLASSES + r]                  (GTS_WANT_BUSY; see above)
+ * Start/finish/digest/cta_sm/busy of a point whose status is not GTS_OK are
  * unspecified.  The digest is sum over v of splitmix64-finalise(
  * (v << 32 | (uint32)start) ^ ((uint64)(uint32)finish * 0x9E3779B97F4A7C15)) mod 2^64.
  * d_scratch (16-byte aligned, scratch_bytes long) is required; see
@@ -200,7 +216,7 @@ gts_status gts_simulate_batch(gts_graph *graph, gts_params *params,
                               uint32_t first_point, uint32_t n_points, uint32_t flags,
                               int32_t *d_start, int32_t *d_finish,
                               int32_t *d_makespan, int32_t *d_status,
-                              uint64_t *d_digest, int32_t *d_cta_sm,
+                              uint64_t *d_digest, int32_t *d_cta_sm, int64_t *d_busy,
                               void *d_scratch, size_t scratch_bytes,
                               void *stream, gts_results **out);
 
@@ -237,7 +253,8 @@ gts_status gts_simulate_batch_noalloc(gts_graph *graph, gts_params *params,
                                       uint32_t first_point, uint32_t n_points, uint32_t flags,
                                       int32_t *d_start, int32_t *d_finish,
                                       int32_t *d_makespan, int32_t *d_status,
-                                      uint64_t *d_digest, int32_t *d_cta_sm, void *stream);
+                                      uint64_t *d_digest, int32_t *d_cta_sm, int64_t *d_busy,
+                                      void *stream);
 
 /* Message for the calling thread's last non-OK host-side status ("" if none). */
 const char *gts_last_error(void);

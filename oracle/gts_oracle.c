@@ -34,6 +34,11 @@
  *   CTA launch latency 0; times are int64 here and any finish above
  *   2^31-1 is reported as overflow.
  *
+ * Busy server-cycles (optional output): for each resource class the sum of
+ * the occupancies of the nodes served by it -- the cycles its servers were
+ * held (Section 5.2).  Utilisation (Section 7.1 reports the tensor cores')
+ * is that divided by servers x makespan.
+ *
  * Plain on purpose: every step scans the resident CTAs, their warp heads and
  * all servers; no heaps, no incremental structures.
  */
@@ -72,11 +77,15 @@ int oracle_simulate(
     const uint8_t *type, const uint16_t *warp, const uint32_t *cta,
     const uint32_t *work, const uint32_t *lat_extra, const uint32_t *cta_kernel,
     const int32_t *prm,
-    int64_t *start, int64_t *finish, int64_t *makespan, int32_t *cta_sm)
+    int64_t *start, int64_t *finish, int64_t *makespan, int32_t *cta_sm,
+    int64_t *busy /* [RC_COUNT + 1]: per-SM classes, then HBM; may be NULL */)
 {
   int64_t v, e, c, w, k, r;
   int status = OR_OK;
   if (n < 0 || m < 0 || n_ctas < 0 || W < 1 || !prm || !makespan) return OR_ERR_INVALID_ARG;
+  int64_t busy_acc[RC_COUNT + 1] = {0, 0, 0, 0, 0, 0};
+  if (busy)
+    for (r = 0; r <= RC_COUNT; r++) busy[r] = 0;
 
   /* ---- parameter row (Table "GPU configurations" quantities) ---- */
   const int64_t num_sms = prm[PR_NUM_SMS], cps = prm[PR_CTAS_PER_SM];
@@ -221,6 +230,8 @@ int oracle_simulate(
         start[v] = t;
         finish[v] = f;
         if (f > mkspan) mkspan = f;
+        if (cls[v] >= 0) busy_acc[cls[v]] += occ[v];
+        if (hocc[v] >= 0) busy_acc[RC_COUNT] += hocc[v];
         if (cls[v] >= 0) { /* take any free server of the class on this SM */
           for (int64_t q = 0; q < cap[cls[v]]; q++) {
             int64_t *s = &srv[cls[v]][sm * cap[cls[v]] + q];
@@ -264,6 +275,8 @@ int oracle_simulate(
     t = tn;
   }
   *makespan = mkspan;
+  if (busy)
+    for (r = 0; r <= RC_COUNT; r++) busy[r] = busy_acc[r];
 
 out:
   free(cls); free(occ); free(hocc); free(lat); free(npend); free(rdy); free(nxt); free(head);

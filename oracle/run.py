@@ -44,7 +44,7 @@ def _load():
             lib = ctypes.CDLL(build())
             p = ctypes.c_void_p
             i64 = ctypes.c_int64
-            lib.oracle_simulate.argtypes = [i64, i64, i64, i64] + [p] * 14
+            lib.oracle_simulate.argtypes = [i64, i64, i64, i64] + [p] * 15
             lib.oracle_simulate.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -57,6 +57,7 @@ class Result:
     start: np.ndarray    # int64 [n]
     finish: np.ndarray   # int64 [n]
     cta_sm: np.ndarray   # int32 [C]
+    busy: np.ndarray = None  # int64 [6]: busy server-cycles of TENSOR, TMA, LSU, ALU, BAR, HBM
 
 
 def _ptr(a):
@@ -81,11 +82,12 @@ def simulate_arrays(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_
     finish = np.empty(max(n, 1), np.int64)
     cta_sm = np.empty(max(C, 1), np.int32)
     mk = ctypes.c_int64(0)
+    busy = np.zeros(6, np.int64)
     st = lib.oracle_simulate(n, m, C, int(warps_per_cta), _ptr(a["row_ptr"]), _ptr(a["col"]), _ptr(a["ekind"]),
                              _ptr(a["type"]), _ptr(a["warp"]), _ptr(a["cta"]), _ptr(a["work"]),
                              _ptr(a["lat_extra"]), _ptr(a["cta_kernel"]), _ptr(prm), _ptr(start), _ptr(finish),
-                             ctypes.byref(mk), _ptr(cta_sm))
-    return Result(int(st), int(mk.value), start[:n], finish[:n], cta_sm[:C])
+                             ctypes.byref(mk), _ptr(cta_sm), _ptr(busy))
+    return Result(int(st), int(mk.value), start[:n], finish[:n], cta_sm[:C], busy)
 
 
 def simulate(graph, params_row) -> Result:

@@ -145,6 +145,27 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
             return -8, 0, start, [None] * n, cta_sm
 
 
+CLASS_ORDER = ("tensor", "tma", "lsu", "alu", "bar", "hbm")
+
+
+def busy_cycles(type_, work, lat_extra, prm, start, makespan):
+    """Busy server-cycles of each class, measured on a finished schedule by
+    sweeping every cycle t in [0, makespan) and counting the servers held at t
+    (a node holds one server of its class on [start, start + occupancy), and
+    one HBM server on [start, start + HBM occupancy)).  Returned in the order
+    TENSOR, TMA, LSU, ALU, BAR, HBM."""
+    prm = [int(x) for x in prm]
+    costs = [node_costs(int(type_[v]), int(work[v]), int(lat_extra[v]), prm) for v in range(len(type_))]
+    total = dict.fromkeys(CLASS_ORDER, 0)
+    for t in range(makespan):
+        for v, (cls, occ, hocc, _lat) in enumerate(costs):
+            if cls is not None and start[v] <= t < start[v] + occ:
+                total[cls] += 1
+            if hocc is not None and start[v] <= t < start[v] + hocc:
+                total["hbm"] += 1
+    return [total[k] for k in CLASS_ORDER]
+
+
 def simulate_graph(g, prm, **kw):
     """Same, for a single workloads.Graph."""
     return simulate(g.row_ptr, g.col, g.ekind, g.type, g.warp, g.cta, g.work, g.lat_extra, g.cta_kernel,

@@ -460,7 +460,7 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
 __global__ void __launch_bounds__(MAX_WPB * 32, 1)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
-           int32_t *d_cta_sm, uint2 *scratch, uint32_t n_warps, uint32_t budget_words) {
+           int32_t *d_cta_sm, int64_t *d_busy, uint2 *scratch, uint32_t n_warps, uint32_t budget_words) {
   extern __shared__ __align__(16) uint32_t smem[];
   const int lane = threadIdx.x & 31;
   const uint32_t wib = threadIdx.x >> 5;
@@ -494,6 +494,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         d_makespan[q] = 0;
         if (want_digest) d_digest[q] = 0;
       }
+      if (d_busy && lane < GTS_BUSY_CLASSES) d_busy[(size_t)q * GTS_BUSY_CLASSES + lane] = 0;
       __syncwarp();
       continue;
     }
@@ -564,6 +565,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     uint32_t issued = 0;
     int32_t mk = 0;
     uint64_t digest = 0;
+    uint64_t busy = 0;  // lane r < 5: server-cycles of per-SM class r; lane 5: HBM
     uint64_t b = INF64;  // this lane's best (effective cycle << 32 | id) over its SMs
     uint32_t bsl = 0;    // ... and its slot
     if (!launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
@@ -614,6 +616,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       const uint64_t f64 = (uint64_t)t + lat;
       if (f64 > 0x7FFFFFFFull) { status = GTS_ERR_OVERFLOW; break; }
       const uint32_t f = (uint32_t)f64;
+      busy += (uint32_t)lane == cls ? occ : ((uint32_t)lane == RC_N ? hocc : 0u);
       cn.x = __shfl_sync(FULL, cn.x, 0);
       cn.y = __shfl_sync(FULL, cn.y, 0);
       // take one free server of the node's class on its SM (lane k tests server k)
@@ -735,6 +738,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       d_makespan[q] = status == GTS_OK ? mk : 0;
       if (want_digest) d_digest[q] = status == GTS_OK ? digest : 0ull;
     }
+    if (d_busy && lane < GTS_BUSY_CLASSES) d_busy[(size_t)q * GTS_BUSY_CLASSES + lane] = status == GTS_OK ? (int64_t)busy : 0;
     __syncwarp();
   }
 }
@@ -1034,18 +1038,21 @@ size_t gts_scratch_bytes(const gts_graph *g, const gts_params *P, uint32_t flags
 
 gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point, uint32_t n_points, uint32_t flags,
                               int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status,
-                              uint64_t *d_digest, int32_t *d_cta_sm, void *d_scratch, size_t scratch_bytes,
-                              void *stream, gts_results **out) {
+                              uint64_t *d_digest, int32_t *d_cta_sm, int64_t *d_busy, void *d_scratch,
+                              size_t scratch_bytes, void *stream, gts_results **out) {
   clear_error();
   if (out) *out = nullptr;
   if (!g || !P || P->graph != g) return fail(GTS_ERR_INVALID_ARG, "null or mismatched graph / params");
-  if (flags & ~(GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM)) return fail(GTS_ERR_INVALID_ARG, "unknown flag");
+  if (flags & ~(GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM | GTS_WANT_BUSY))
+    return fail(GTS_ERR_INVALID_ARG, "unknown flag");
   if ((uint64_t)first_point + n_points > P->n_points) return fail(GTS_ERR_INVALID_ARG, "point range outside the table");
   if (!d_makespan || !d_status) return fail(GTS_ERR_INVALID_ARG, "d_makespan and d_status are required");
   if ((flags & GTS_FULL_TRACE) && g->dg.row_nodes && (!d_start || !d_finish))
     return fail(GTS_ERR_INVALID_ARG, "FULL_TRACE needs d_start and d_finish");
   if ((flags & GTS_WANT_DIGEST) && !d_digest) return fail(GTS_ERR_INVALID_ARG, "WANT_DIGEST needs d_digest");
   if ((flags & GTS_WANT_CTA_SM) && g->dg.row_ctas && !d_cta_sm) return fail(GTS_ERR_INVALID_ARG, "WANT_CTA_SM needs d_cta_sm");
+  if ((flags & GTS_WANT_BUSY) && !d_busy) return fail(GTS_ERR_INVALID_ARG, "WANT_BUSY needs d_busy");
+  if ((flags & GTS_WANT_BUSY) && (uintptr_t)d_busy % 8 != 0) return fail(GTS_ERR_INVALID_ARG, "d_busy must be 8-byte aligned");
   if (!d_scratch) return fail(GTS_ERR_NOMEM, "scratch required (gts_scratch_bytes)");
   if ((uintptr_t)d_scratch % 16 != 0) return fail(GTS_ERR_INVALID_ARG, "scratch must be 16-byte aligned");
   cudaStream_t s = (cudaStream_t)stream;
@@ -1056,7 +1063,7 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
     k_simulate<<<pl.blocks, pl.wpb * 32, pl.smem, s>>>(
         g->dg, P->d_params, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status,
         (flags & GTS_WANT_DIGEST) ? d_digest : nullptr, (flags & GTS_WANT_CTA_SM) ? d_cta_sm : nullptr,
-        (uint2 *)d_scratch, pl.warps, pl.words);
+        (flags & GTS_WANT_BUSY) ? d_busy : nullptr, (uint2 *)d_scratch, pl.warps, pl.words);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "simulate: launch");
   }
@@ -1136,7 +1143,8 @@ extern "C" {
 
 gts_status gts_simulate_batch_noalloc(gts_graph *g, gts_params *P, uint32_t first_point, uint32_t n_points,
                                       uint32_t flags, int32_t *d_start, int32_t *d_finish, int32_t *d_makespan,
-                                      int32_t *d_status, uint64_t *d_digest, int32_t *d_cta_sm, void *stream) {
+                                      int32_t *d_status, uint64_t *d_digest, int32_t *d_cta_sm, int64_t *d_busy,
+                                      void *stream) {
   clear_error();
   if (!g) return fail(GTS_ERR_INVALID_ARG, "null graph");
   if (scratch_row_bytes(g) > GTS_STATIC_SCRATCH_BYTES)
@@ -1146,7 +1154,7 @@ gts_status gts_simulate_batch_noalloc(gts_graph *g, gts_params *P, uint32_t firs
   gts_status st = static_scratch(&scr);
   if (st != GTS_OK) return st;
   return gts_simulate_batch(g, P, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status, d_digest,
-                            d_cta_sm, scr, GTS_STATIC_SCRATCH_BYTES, stream, nullptr);
+                            d_cta_sm, d_busy, scr, GTS_STATIC_SCRATCH_BYTES, stream, nullptr);
 }
 
 }  // extern "C"

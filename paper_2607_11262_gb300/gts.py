@@ -32,6 +32,11 @@ GTS_ERR_UNSUPPORTED = -9
 GTS_FULL_TRACE = 1
 GTS_WANT_DIGEST = 2
 GTS_WANT_CTA_SM = 4
+GTS_WANT_BUSY = 8
+
+GTS_BUSY_CLASSES = 6
+GTS_BUSY_TENSOR, GTS_BUSY_TMA, GTS_BUSY_LSU, GTS_BUSY_ALU, GTS_BUSY_BAR, GTS_BUSY_HBM = range(6)
+BUSY_NAMES = ("tensor", "tma", "lsu", "alu", "bar", "hbm")
 
 GTS_STATIC_SCRATCH_BYTES = 32 << 20
 
@@ -85,13 +90,13 @@ def load():
     lib.gts_row_ctas.restype = u32
     lib.gts_scratch_bytes.argtypes = [vp, vp, u32]
     lib.gts_scratch_bytes.restype = sz
-    lib.gts_simulate_batch.argtypes = [vp, vp, u32, u32, u32, vp, vp, vp, vp, vp, vp, vp, sz, vp, pp]
+    lib.gts_simulate_batch.argtypes = [vp, vp, u32, u32, u32, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp, pp]
     lib.gts_simulate_batch.restype = i32
     lib.gts_read_results.argtypes = [vp, vp, vp, vp, u32]
     lib.gts_read_results.restype = i32
     lib.gts_results_destroy.argtypes = [vp]
     lib.gts_results_destroy.restype = i32
-    lib.gts_simulate_batch_noalloc.argtypes = [vp, vp, u32, u32, u32, vp, vp, vp, vp, vp, vp, vp]
+    lib.gts_simulate_batch_noalloc.argtypes = [vp, vp, u32, u32, u32, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.gts_simulate_batch_noalloc.restype = i32
     lib.gts_last_error.argtypes = []
     lib.gts_last_error.restype = ctypes.c_char_p
@@ -142,10 +147,10 @@ def gts_scratch_bytes(graph, params, flags):
 
 
 def gts_simulate_batch(graph, params, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status,
-                       d_digest, d_cta_sm, d_scratch, scratch_bytes, stream=0, want_handle=False):
+                       d_digest, d_cta_sm, d_busy, d_scratch, scratch_bytes, stream=0, want_handle=False):
     h = ctypes.c_void_p()
     _check(load().gts_simulate_batch(graph, params, first_point, n_points, flags, d_start, d_finish, d_makespan,
-                                     d_status, d_digest, d_cta_sm, d_scratch, scratch_bytes, stream,
+                                     d_status, d_digest, d_cta_sm, d_busy, d_scratch, scratch_bytes, stream,
                                      ctypes.byref(h) if want_handle else None))
     return h.value if want_handle else None
 
@@ -159,11 +164,11 @@ def gts_results_destroy(results):
 
 
 def gts_simulate_batch_noalloc(graph, params, first_point, n_points, flags, d_start, d_finish, d_makespan,
-                               d_status, d_digest, d_cta_sm, stream=0):
+                               d_status, d_digest, d_cta_sm, d_busy, stream=0):
     """gts_simulate_batch without caller scratch: libgts uses its own fixed
     device array (GTS_STATIC_SCRATCH_BYTES) and allocates nothing."""
     _check(load().gts_simulate_batch_noalloc(graph, params, first_point, n_points, flags, d_start, d_finish,
-                                             d_makespan, d_status, d_digest, d_cta_sm, stream))
+                                             d_makespan, d_status, d_digest, d_cta_sm, d_busy, stream))
 
 
 def gts_last_error():
@@ -282,6 +287,7 @@ class BatchOutput:
     finish: object = None
     digest: object = None
     cta_sm: object = None
+    busy: object = None
 
 
 def alloc_outputs(dgraph: DeviceGraph, n_points: int, flags: int):
@@ -296,6 +302,8 @@ def alloc_outputs(dgraph: DeviceGraph, n_points: int, flags: int):
         out.digest = torch.empty(n_points, dtype=torch.int64, device=dev)
     if flags & GTS_WANT_CTA_SM:
         out.cta_sm = torch.empty((n_points, dgraph.row_ctas), dtype=torch.int32, device=dev)
+    if flags & GTS_WANT_BUSY:
+        out.busy = torch.empty((n_points, GTS_BUSY_CLASSES), dtype=torch.int64, device=dev)
     return out
 
 
@@ -317,7 +325,23 @@ def simulate(dgraph: DeviceGraph, dparams: DeviceParams, first_point=0, n_points
         scratch = torch.empty(max(nb, 16), dtype=torch.uint8, device=dgraph.workspace.device)
     gts_simulate_batch(dgraph.handle, dparams.handle, first_point, n_points, flags, _ptr(out.start),
                        _ptr(out.finish), _ptr(out.makespan), _ptr(out.status), _ptr(out.digest),
-                       _ptr(out.cta_sm), _ptr(scratch), 0 if scratch is None else scratch.numel(),
+                       _ptr(out.cta_sm), _ptr(out.busy), _ptr(scratch), 0 if scratch is None else scratch.numel(),
                        _stream_handle(stream))
     out.scratch = scratch
     return out
+
+
+def utilisation(busy, makespan, params):
+    """Per-class utilisation of each point from its busy server-cycles:
+    busy_r / (servers_r * makespan), servers_r = cap_r * num_sms for the per-SM
+    classes and cap_hbm for HBM; 0 where the makespan is 0.  numpy in, numpy out
+    ([n_points][GTS_BUSY_CLASSES] float64)."""
+    import numpy as np
+    busy = np.asarray(busy, np.float64)
+    prm = np.asarray(params, np.int64)
+    mk = np.asarray(makespan, np.float64)
+    servers = np.empty((prm.shape[0], GTS_BUSY_CLASSES), np.float64)
+    servers[:, :5] = prm[:, 13:18] * prm[:, 0:1]
+    servers[:, 5] = prm[:, 18]
+    den = servers * mk[:, None]
+    return np.divide(busy, den, out=np.zeros_like(busy), where=den > 0)

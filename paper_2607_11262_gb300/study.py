@@ -1,0 +1,82 @@
+"""Software-pipelining case study and tile-graph ablation on the GPU
+(Section 7.1 "Software Pipelining Impact"; Section 6.4 ablation).
+
+Every (organisation, tile, ablation) graph of ``pipelines.study_set`` runs on
+one simulated Hopper SM through libgts; the table reports, per graph, the
+makespan, the tensor-pipe utilisation (busy tensor cycles / makespan, from the
+engine's busy-cycle output) and the performance normalised to the fastest
+organisation of the same tile.  With ``--points-per-graph`` > 1 the extra
+design points sweep DRAM bandwidth and tensor rate, and the table adds the
+utilisation range over the sweep.
+
+    python -m paper_2607_11262_gb300.study [--points-per-graph 64] [--json out.json]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import numpy as np
+
+from . import gts, pipelines
+
+
+def run_study(points_per_graph=1, device="cuda"):
+    """Runs the study; returns a list of dicts, one per graph, in stacking order."""
+    import torch
+    gts.load()
+    graph, cases = pipelines.study_set()
+    params = pipelines.study_params(len(cases), points_per_graph)
+    dg = gts.DeviceGraph(graph, device=device)
+    dp = gts.DeviceParams(dg, params)
+    out = gts.simulate(dg, dp, flags=gts.GTS_WANT_BUSY)
+    torch.cuda.synchronize()
+    status = out.status.cpu().numpy()
+    if np.any(status != gts.GTS_OK):
+        raise gts.GtsError(int(status[status != 0][0]), "a study point did not simulate")
+    mk = out.makespan.cpu().numpy()
+    busy = out.busy.cpu().numpy()
+    util = gts.utilisation(busy, mk, params)[:, gts.GTS_BUSY_TENSOR]
+    dp.close()
+    dg.close()
+    rows = []
+    for i, (org, tile, abl) in enumerate(cases):
+        sl = slice(i * points_per_graph, (i + 1) * points_per_graph)
+        rows.append(dict(org=org, tile=list(tile), ablation=abl, makespan=int(mk[sl][0]),
+                         tensor_util=float(util[sl][0]), tensor_busy=int(busy[sl][0, gts.GTS_BUSY_TENSOR]),
+                         tma_busy=int(busy[sl][0, gts.GTS_BUSY_TMA]),
+                         util_min=float(util[sl].min()), util_max=float(util[sl].max())))
+    best = {}
+    for r in rows:
+        if r["ablation"] == "full":
+            k = tuple(r["tile"])
+            best[k] = min(best.get(k, r["makespan"]), r["makespan"])
+    for r in rows:
+        r["normalised_perf"] = best[tuple(r["tile"])] / r["makespan"]
+    return rows
+
+
+def format_table(rows):
+    lines = [f"{'organisation':<16}{'tile':<15}{'ablation':<11}{'makespan':>10}{'perf':>7}{'tensor':>8}"
+             f"{'sweep':>15}"]
+    for r in rows:
+        tile = "x".join(str(x) for x in r["tile"])
+        lines.append(f"{r['org']:<16}{tile:<15}{r['ablation']:<11}{r['makespan']:>10d}{r['normalised_perf']:>7.3f}"
+                     f"{100 * r['tensor_util']:>7.1f}%{100 * r['util_min']:>7.1f}-{100 * r['util_max']:.1f}%")
+    return "\n".join(lines)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--points-per-graph", type=int, default=1)
+    ap.add_argument("--json", default=None)
+    args = ap.parse_args()
+    rows = run_study(args.points_per_graph)
+    print(format_table(rows))
+    if args.json:
+        with open(args.json, "w") as f:
+            json.dump(rows, f, indent=1)
+
+
+if __name__ == "__main__":
+    main()

@@ -668,6 +668,12 @@ def workload(name: str, points: int | None = None, instances: int | None = None)
         g = stress_set(k)
         p = stress_params(k)
         d = f"{k} random layered DAGs x 100k nodes, 64 layers, fan-in 1-4, latency 4-4096"
+    elif name == "pipelines":
+        from . import pipelines
+        g, cases = pipelines.study_set()
+        p = pipelines.study_params(len(cases), 64)
+        d = (f"GEMM+SiLU pipeline study: 4 organisations x {len(pipelines.TILES)} tiles x 4 ablations, "
+             "10 waves on 1 SM; 64 points per graph (DRAM and tensor rate swept)")
     else:
         raise KeyError(name)
     if points is not None:
@@ -676,3 +682,4 @@ def workload(name: str, points: int | None = None, instances: int | None = None)
 
 
 WORKLOADS = ("gemm512", "wsgemm8192", "fa_fwd", "decoder", "stress")
+STUDIES = ("pipelines",)

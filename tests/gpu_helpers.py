@@ -25,7 +25,7 @@ def run_gpu(graph, params, flags=None, first_point=0, n_points=None):
 
     from paper_2607_11262_gb300 import gts
     if flags is None:
-        flags = gts.GTS_FULL_TRACE | gts.GTS_WANT_DIGEST | gts.GTS_WANT_CTA_SM
+        flags = gts.GTS_FULL_TRACE | gts.GTS_WANT_DIGEST | gts.GTS_WANT_CTA_SM | gts.GTS_WANT_BUSY
     dg = gts.DeviceGraph(graph)
     dp = gts.DeviceParams(dg, params)
     out = gts.simulate(dg, dp, first_point=first_point, n_points=n_points, flags=flags)
@@ -38,6 +38,8 @@ def run_gpu(graph, params, flags=None, first_point=0, n_points=None):
         res["digest"] = out.digest.cpu().numpy().astype(np.uint64)
     if out.cta_sm is not None:
         res["cta_sm"] = out.cta_sm.cpu().numpy()
+    if out.busy is not None:
+        res["busy"] = out.busy.cpu().numpy()
     del out
     dp.close()
     dg.close()
@@ -70,3 +72,5 @@ def assert_point_equal(graph, params, res, q, ref, check_trace=True):
         assert np.array_equal(res["cta_sm"][q][:c], ref.cta_sm), q
     if "digest" in res:
         assert int(res["digest"][q]) == digest(ref.start, ref.finish), q
+    if "busy" in res:
+        assert list(res["busy"][q]) == list(ref.busy), (q, list(res["busy"][q]), list(ref.busy))

@@ -49,7 +49,7 @@ def test_binding_loads_and_sizes_without_gpu(lib):
     assert gts.gts_graph_workspace_bytes(10, 12, 2, 3, 0) == 0       # no graph
     assert gts.load().gts_graph_create(None, None, None) == gts.GTS_ERR_INVALID_ARG
     assert "null" in gts.gts_last_error()
-    assert gts.load().gts_simulate_batch(None, None, 0, 0, 0, None, None, None, None, None, None, None, 0,
+    assert gts.load().gts_simulate_batch(None, None, 0, 0, 0, None, None, None, None, None, None, None, None, 0,
                                          None, None) == gts.GTS_ERR_INVALID_ARG
 
 

@@ -41,7 +41,7 @@ def test_full_size_workload(gts_mod, name, k):
     w = W.workload(name)
     dg = gts.DeviceGraph(w.graph)
     dp = gts.DeviceParams(dg, w.params)
-    flags = gts.GTS_FULL_TRACE | gts.GTS_WANT_DIGEST | gts.GTS_WANT_CTA_SM
+    flags = gts.GTS_FULL_TRACE | gts.GTS_WANT_DIGEST | gts.GTS_WANT_CTA_SM | gts.GTS_WANT_BUSY
     out = gts.simulate(dg, dp, flags=flags)
     torch.cuda.synchronize()
     status = out.status.cpu().numpy()
@@ -63,9 +63,10 @@ def test_full_size_workload(gts_mod, name, k):
     finish = out.finish.index_select(0, sel).cpu().numpy()
     cta_sm = out.cta_sm.index_select(0, sel).cpu().numpy()
     digest = out.digest.cpu().numpy().astype(np.uint64)
+    busy = out.busy.cpu().numpy()
     for j, p in enumerate(pts):
         one = {"status": res["status"][[p]], "makespan": res["makespan"][[p]], "start": start[[j]],
-               "finish": finish[[j]], "cta_sm": cta_sm[[j]], "digest": digest[[p]]}
+               "finish": finish[[j]], "cta_sm": cta_sm[[j]], "digest": digest[[p]], "busy": busy[[p]]}
         H.assert_point_equal(w.graph, w.params[p], one, 0, refs[p])
     del out
     dp.close()

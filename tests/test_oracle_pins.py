@@ -9,6 +9,9 @@
   makespan; finish = start + latency; no unit over capacity at any cycle; warp
   starts are non-decreasing; Graham's (2 - 1/m) bound against a brute-force
   optimum of P|prec|Cmax;
+* busy server-cycles: equal to the stepper's cycle-by-cycle count of held
+  servers; a single saturated server is busy for the whole makespan; busy
+  cycles never exceed servers x makespan;
 * error statuses.
 """
 import json
@@ -28,19 +31,23 @@ KIND = {"DATA": W.DATA, "ISSUE": W.ISSUE}
 
 
 def both(g, prm):
+    """Oracle result and the stepper's (status, makespan, start, finish, cta_sm,
+    busy cycles counted cycle by cycle)."""
     r = run.simulate(g, prm)
     s = stepper.simulate_graph(g, prm)
-    return r, s
+    busy = stepper.busy_cycles(g.type, g.work, g.lat_extra, prm, s[2], s[1]) if s[0] == 0 else None
+    return r, s + (busy,)
 
 
 def assert_same(r, s):
-    st, mk, start, fin, cta_sm = s
+    st, mk, start, fin, cta_sm, busy = s
     assert r.status == st
     if st == 0:
         assert r.makespan == mk
         assert list(r.start) == start
         assert list(r.finish) == fin
         assert list(r.cta_sm) == cta_sm
+        assert list(r.busy) == busy
 
 
 # ------------------------------------------------------------------ golden
@@ -197,6 +204,8 @@ def test_single_server_no_idle():
         r = run.simulate(g, TG.unit_params(1, 1, 1, 1))
         assert r.status == 0
         assert r.makespan == int(g.work.sum())
+        assert r.busy[0] == r.makespan          # the tensor server never idles
+        assert list(r.busy[1:]) == [0] * 5
 
 
 # ------------------------------------------------------------------ bounds and invariants
@@ -262,6 +271,13 @@ def test_invariants_random_graphs():
                 work[(sm[v], c)] = work.get((sm[v], c), 0) + o
         assert all(w <= caps * r.makespan for w in work.values())
         assert sum(o[2] for o in occ if o[2] is not None) <= cap_hbm * r.makespan
+        # busy server-cycles: per class the unit-rate occupancies; within capacity
+        names = ("tensor", "tma", "lsu", "alu", "bar")
+        for k, c in enumerate(names):
+            assert r.busy[k] == sum(o[1] for o in occ if o[0] == c)
+        assert r.busy[5] == sum(o[2] for o in occ if o[2] is not None)
+        assert all(r.busy[k] <= caps * int(prm[0]) * r.makespan for k in range(5))
+        assert r.busy[5] <= cap_hbm * r.makespan
 
 
 def _opt_makespan(p, preds, m):

@@ -14,7 +14,7 @@ from tests import tinygraphs as TG
 
 pytestmark = pytest.mark.gpu
 
-FLAGS = 1 | 2 | 4  # full trace, digest, CTA placement
+FLAGS = 1 | 2 | 4 | 8  # full trace, digest, CTA placement, busy cycles
 
 
 @pytest.fixture(scope="module")
@@ -32,11 +32,11 @@ def _noalloc(gts, dg, dp, out, first=0, n=None):
     n = dp.n_points - first if n is None else n
     p = lambda t: 0 if t is None else t.data_ptr()  # noqa: E731
     gts.gts_simulate_batch_noalloc(dg.handle, dp.handle, first, n, FLAGS, p(out.start), p(out.finish),
-                                   p(out.makespan), p(out.status), p(out.digest), p(out.cta_sm),
+                                   p(out.makespan), p(out.status), p(out.digest), p(out.cta_sm), p(out.busy),
                                    torch.cuda.current_stream().cuda_stream)
     torch.cuda.synchronize()
     return {k: getattr(out, k).cpu().numpy().copy() for k in ("makespan", "status", "start", "finish", "digest",
-                                                               "cta_sm")}
+                                                               "cta_sm", "busy")}
 
 
 def _reference(gts, dg, dp):
@@ -44,7 +44,7 @@ def _reference(gts, dg, dp):
     out = gts.simulate(dg, dp, flags=FLAGS)
     torch.cuda.synchronize()
     return {k: getattr(out, k).cpu().numpy().copy() for k in ("makespan", "status", "start", "finish", "digest",
-                                                               "cta_sm")}
+                                                               "cta_sm", "busy")}
 
 
 def _same(a, b):
@@ -96,6 +96,6 @@ def test_noalloc_partial_range_and_too_large(gts_mod):
     outb = gts.alloc_outputs(dgb, 1, 0)
     with pytest.raises(gts.GtsError) as e:
         gts.gts_simulate_batch_noalloc(dgb.handle, dpb.handle, 0, 1, 0, 0, 0, outb.makespan.data_ptr(),
-                                       outb.status.data_ptr(), 0, 0, 0)
+                                       outb.status.data_ptr(), 0, 0, 0, 0)
     assert e.value.status == gts.GTS_ERR_NOMEM
     assert "static scratch" in gts.gts_last_error()
