@@ -7,7 +7,7 @@ makespan, the tensor-pipe utilisation (busy tensor cycles / makespan, from the
 engine's busy-cycle output) and the performance normalised to the fastest
 organisation of the same tile.  With ``--points-per-graph`` > 1 the extra
 design points sweep DRAM bandwidth and tensor rate, and the table adds the
-utilisation range over the sweep.
+utilisation's minimum, mean and maximum over the sweep.
 
     python -m paper_2607_11262_gb300.study [--points-per-graph 64] [--json out.json]
 """
@@ -45,7 +45,8 @@ def run_study(points_per_graph=1, device="cuda"):
         rows.append(dict(org=org, tile=list(tile), ablation=abl, makespan=int(mk[sl][0]),
                          tensor_util=float(util[sl][0]), tensor_busy=int(busy[sl][0, gts.GTS_BUSY_TENSOR]),
                          tma_busy=int(busy[sl][0, gts.GTS_BUSY_TMA]),
-                         util_min=float(util[sl].min()), util_max=float(util[sl].max())))
+                         util_min=float(util[sl].min()), util_mean=float(util[sl].mean()),
+                         util_max=float(util[sl].max())))
     best = {}
     for r in rows:
         if r["ablation"] == "full":
@@ -58,11 +59,12 @@ def run_study(points_per_graph=1, device="cuda"):
 
 def format_table(rows):
     lines = [f"{'organisation':<16}{'tile':<15}{'ablation':<11}{'makespan':>10}{'perf':>7}{'tensor':>8}"
-             f"{'sweep':>15}"]
+             f"{'sweep min/mean/max':>22}"]
     for r in rows:
         tile = "x".join(str(x) for x in r["tile"])
         lines.append(f"{r['org']:<16}{tile:<15}{r['ablation']:<11}{r['makespan']:>10d}{r['normalised_perf']:>7.3f}"
-                     f"{100 * r['tensor_util']:>7.1f}%{100 * r['util_min']:>7.1f}-{100 * r['util_max']:.1f}%")
+                     f"{100 * r['tensor_util']:>7.1f}%{100 * r['util_min']:>8.1f}/{100 * r['util_mean']:.1f}/"
+                     f"{100 * r['util_max']:.1f}%")
     return "\n".join(lines)
 
 

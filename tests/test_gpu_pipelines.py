@@ -47,6 +47,7 @@ def test_study_table_matches_oracle(gts_mod):
         assert r["tensor_util"] == pytest.approx(utils[0], rel=1e-12)
         assert r["util_min"] == pytest.approx(min(utils), rel=1e-12)
         assert r["util_max"] == pytest.approx(max(utils), rel=1e-12)
+        assert r["util_mean"] == pytest.approx(sum(utils) / 3, rel=1e-12)
     assert max(r["normalised_perf"] for r in rows if r["ablation"] == "full") == 1.0
 
 
