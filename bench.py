@@ -123,7 +123,10 @@ def dist_env():
     return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
 
 
-def load_workload(name, rank, points):
+POLICIES = {"lowest_id": 0, "gto": 1, "rr": 2}
+
+
+def load_workload(name, rank, points, policy="lowest_id", subpartitions=4):
     from paper_2607_11262_gb300 import workloads as W
     w = W.workload(name)
     if rank > 0 and name == "pipelines":
@@ -138,7 +141,19 @@ def load_workload(name, rank, points):
         w.params = W.sweep_params(W.SEED0 + 100 * rank + W.WORKLOADS.index(name) + 1, w.params.shape[0], axes, cps)
     if points is not None:
         w.params = w.params[:points]
+    w.params = np.ascontiguousarray(w.params)
+    w.params[:, W.P_ISSUE_POLICY] = POLICIES[policy]
+    w.params[:, W.P_SUBPARTITIONS] = 0 if policy == "lowest_id" else subpartitions
     return w
+
+
+def workload_config(w, args, world):
+    """The ``config`` object both arms print for a workload."""
+    return {"workload": w.name, "description": w.description, "nodes": w.graph.max_graph_nodes,
+            "edges": w.graph.n_edges, "design_points_per_gpu": int(w.params.shape[0]), "full_trace": True,
+            "issue_policy": args.policy, "subpartitions": 0 if args.policy == "lowest_id" else args.subpartitions,
+            "l2": "inputs+outputs larger than L2 (trace rows alone exceed it)",
+            "parallelism": f"design points sharded over {world} GPU(s)"}
 
 
 def cpu_baseline(graph, params, seconds=15.0, procs=None):
@@ -167,7 +182,7 @@ def run_reference(args):
     ws, rank, _ = dist_env()
     if rank != 0:
         return
-    w = load_workload(args.workload, 0, args.points)
+    w = load_workload(args.workload, 0, args.points, args.policy, args.subpartitions)
     g = w.graph
     vals, times = [], []
     node_points = node_points_of(g, w.params)
@@ -177,12 +192,10 @@ def run_reference(args):
             vals.append(cb["value"])
             times.append(cb)
     v = float(np.median(vals))
-    n = g.max_graph_nodes
     line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": node_points / v * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-            "config": {"workload": w.name, "description": w.description, "nodes": n,
-                       "design_points": int(w.params.shape[0])},
+            "config": workload_config(w, args, ws),
             "impl": "reference", "cpu_baseline": dict(times[-1], value=v),
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -196,6 +209,8 @@ def main():
     ap.add_argument("--impl", default="gts", choices=["gts", "reference"])
     ap.add_argument("--workload", default="wsgemm8192")
     ap.add_argument("--points", type=int, default=None)
+    ap.add_argument("--policy", default="lowest_id", choices=sorted(POLICIES))
+    ap.add_argument("--subpartitions", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ref-seconds", type=float, default=15.0)
     args = ap.parse_args()
@@ -211,10 +226,9 @@ def main():
     from paper_2607_11262_gb300 import gts
     gts.load()
 
-    w = load_workload(args.workload, rank, args.points)
+    w = load_workload(args.workload, rank, args.points, args.policy, args.subpartitions)
     g = w.graph
     P = int(w.params.shape[0])
-    n = g.max_graph_nodes
     node_points = node_points_of(g, w.params)
     flags = gts.GTS_FULL_TRACE
     stream = torch.cuda.Stream()
@@ -279,10 +293,7 @@ def main():
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "int32", "data": "synthetic",
-        "config": {"workload": w.name, "description": w.description, "nodes": n, "edges": g.n_edges,
-                   "design_points_per_gpu": P, "full_trace": True,
-                   "l2": "inputs+outputs larger than L2 (trace rows alone exceed it)",
-                   "parallelism": f"design points sharded over {ws} GPU(s)"},
+        "config": workload_config(w, args, ws),
         "design_points_per_s": P * ws / kernel_s,
         "hbm_gbs_algorithmic": achieved,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

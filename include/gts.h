@@ -80,7 +80,7 @@ typedef int32_t gts_status;
 
 /* Parameter row: GTS_NPARAM int32 per design point (Table "GPU configurations"
  * quantities in cycles and bytes/FMAs/ops per cycle). */
-#define GTS_NPARAM 24
+#define GTS_NPARAM 32
 #define GTS_P_NUM_SMS      0
 #define GTS_P_CTAS_PER_SM  1
 #define GTS_P_HBM_BPC      2   /* global DRAM bytes per cycle (one HBM server) */
@@ -101,7 +101,31 @@ typedef int32_t gts_status;
 #define GTS_P_CAP_BAR     17
 #define GTS_P_CAP_HBM     18   /* global HBM servers */
 #define GTS_P_GRAPH_INDEX 19   /* which graph of a stacked set this point runs */
-/* 20..23 reserved, must be 0 */
+#define GTS_P_ISSUE_POLICY 20  /* GTS_POLICY_*, see below */
+#define GTS_P_SUBPARTITIONS 21 /* issue schedulers per SM: 1..32 for GTO / RR, 0 for LOWEST_ID */
+/* 22..31 reserved, must be 0 */
+
+/*
+ * Issue policies (Section 5.3: ready nodes sit in per-subpartition queues
+ * served by greedy-then-oldest or round-robin schedulers).
+ *  GTS_POLICY_LOWEST_ID: one global order -- at each cycle, the lowest node id
+ *    among issuable warp heads issues, one at a time, until none is left; no
+ *    per-cycle issue limit.
+ *  GTS_POLICY_GTO / GTS_POLICY_RR: every SM has `subpartitions` schedulers.
+ *    The warp slot l = (CTA's slot on its SM) * warps_per_cta + warp belongs to
+ *    scheduler l mod subpartitions.  A scheduler issues at most one node per
+ *    cycle: among its issuable warp heads, the first in its order --
+ *      GTO: the slot it issued from last (greedy) if issuable, else the oldest
+ *           warp (lowest CTA id * warps_per_cta + warp);
+ *      RR:  slots in cyclic order starting after the slot it issued from last
+ *           (from slot 0 before its first issue).
+ *    Within a cycle the schedulers' picks issue in ascending node id, one at a
+ *    time, each followed by the state update, until no scheduler that has not
+ *    issued in this cycle has an issuable head.
+ */
+#define GTS_POLICY_LOWEST_ID 0
+#define GTS_POLICY_GTO       1
+#define GTS_POLICY_RR        2
 
 /* Flags of gts_simulate_batch. */
 #define GTS_FULL_TRACE  1u  /* write d_start / d_finish [n_points][row_nodes] */

@@ -26,6 +26,14 @@
  *   - The issue scheduler picks, at the current cycle t, the LOWEST node id
  *     among issuable warp heads, one node at a time, launching CTAs first,
  *     until nothing changes at t; then t jumps to the next event time.
+ *   - Optional per-subpartition schedulers (Section 5.3: per-subpartition
+ *     queues under greedy-then-oldest or round-robin): each SM has nsub
+ *     schedulers; warp slot l = (CTA's slot on its SM) * W + warp belongs to
+ *     scheduler l mod nsub, which issues at most one node per cycle -- the
+ *     first of its issuable heads in policy order (GTO: the slot it issued
+ *     from last, then the oldest warp, CTA id * W + warp; RR: cyclic slot
+ *     order after its last slot).  The schedulers' picks go in ascending node
+ *     id, one at a time.
  *
  * Readings where the paper is silent (the framework's fixed choices):
  *   lowest-id issue in place of GTO/round-robin; an ISSUE edge lets the
@@ -64,8 +72,9 @@ enum {
   PR_NUM_SMS = 0, PR_CTAS_PER_SM, PR_HBM_BPC, PR_DRAM_LAT, PR_TMA_BPC, PR_TMA_LAT,
   PR_SMEM_BPC, PR_SMEM_LAT, PR_MMA_FMA_PC, PR_MMA_LAT, PR_ALU_OPS_PC, PR_ALU_LAT,
   PR_BAR_LAT, PR_CAP_TENSOR, PR_CAP_TMA, PR_CAP_LSU, PR_CAP_ALU, PR_CAP_BAR,
-  PR_CAP_HBM, PR_GRAPH_INDEX, PR_COUNT = 24
+  PR_CAP_HBM, PR_GRAPH_INDEX, PR_ISSUE_POLICY, PR_SUBPARTITIONS, PR_COUNT = 32
 };
+enum { POL_LOWEST_ID = 0, POL_GTO = 1, POL_RR = 2 };
 
 #define INT32_LIMIT ((int64_t)2147483647)
 
@@ -98,6 +107,18 @@ int oracle_simulate(
   if (prm[PR_DRAM_LAT] < 0 || prm[PR_TMA_LAT] < 0 || prm[PR_SMEM_LAT] < 0 || prm[PR_MMA_LAT] < 0 ||
       prm[PR_ALU_LAT] < 0 || prm[PR_BAR_LAT] < 0)
     return OR_ERR_INVALID_PARAMS;
+  const int64_t policy = prm[PR_ISSUE_POLICY], nsub = prm[PR_SUBPARTITIONS];
+  if (policy == POL_LOWEST_ID) {
+    if (nsub != 0) return OR_ERR_INVALID_PARAMS;
+  } else if (policy == POL_GTO || policy == POL_RR) {
+    if (nsub < 1 || nsub > 32) return OR_ERR_INVALID_PARAMS;
+  } else {
+    return OR_ERR_INVALID_PARAMS;
+  }
+  for (k = PR_SUBPARTITIONS + 1; k < PR_COUNT; k++)
+    if (prm[k] != 0) return OR_ERR_INVALID_PARAMS;
+  const int64_t per = cps * W;               /* warp slots per SM */
+  const int64_t nq = num_sms * (nsub ? nsub : 1);
 
   /* ---- graph contract ---- */
   if (row_ptr[0] != 0 || (int64_t)row_ptr[n] != m) return OR_ERR_INVALID_GRAPH;
@@ -124,11 +145,16 @@ int oracle_simulate(
   int64_t *sm_of = malloc(sizeof(int64_t) * (size_t)(n_ctas ? n_ctas : 1));
   int64_t *res = malloc(sizeof(int64_t) * (size_t)(n_ctas ? n_ctas : 1)); /* launched, not yet seen retired */
   int64_t *res_cnt = malloc(sizeof(int64_t) * (size_t)num_sms);
+  int64_t *slot_of = malloc(sizeof(int64_t) * (size_t)(n_ctas ? n_ctas : 1)); /* CTA's slot on its SM */
+  int64_t *sub_avail = calloc((size_t)nq, sizeof(int64_t)); /* scheduler may issue from this cycle on */
+  int64_t *sub_last = malloc(sizeof(int64_t) * (size_t)nq);  /* warp slot it issued from last, -1 none */
+  int64_t *cand = malloc(sizeof(int64_t) * (size_t)nq);
+  int64_t *cand_key = malloc(sizeof(int64_t) * (size_t)nq);
   int64_t *srv[RC_COUNT];
   int64_t *hsrv = calloc((size_t)cap_hbm, sizeof(int64_t));
   for (r = 0; r < RC_COUNT; r++) srv[r] = calloc((size_t)(num_sms * cap[r]), sizeof(int64_t));
   int nomem = !cls || !occ || !hocc || !lat || !npend || !rdy || !nxt || !head || !rem || !endt ||
-              !sm_of || !res || !res_cnt || !hsrv;
+              !sm_of || !res || !res_cnt || !hsrv || !slot_of || !sub_avail || !sub_last || !cand || !cand_key;
   for (r = 0; r < RC_COUNT; r++) nomem |= !srv[r];
   if (nomem) { status = OR_ERR_NOMEM; goto out; }
 
@@ -164,7 +190,8 @@ int oracle_simulate(
   for (v = 0; v < n; v++)
     for (e = row_ptr[v]; e < (int64_t)row_ptr[v + 1]; e++) npend[col[e]]++;
   for (v = 0; v < n; v++) rem[cta[v]]++;
-  for (c = 0; c < n_ctas; c++) { sm_of[c] = -1; if (cta_sm) cta_sm[c] = -1; }
+  for (c = 0; c < n_ctas; c++) { sm_of[c] = -1; slot_of[c] = -1; if (cta_sm) cta_sm[c] = -1; }
+  for (k = 0; k < nq; k++) sub_last[k] = -1;
   for (v = 0; v < n; v++) { start[v] = -1; finish[v] = -1; }
 
   int64_t t = 0, issued = 0, next_cta = 0, nres = 0, mkspan = 0;
@@ -193,19 +220,31 @@ int oracle_simulate(
         for (k = 0; k < num_sms; k++)
           if (res_cnt[k] < cps) { sm = k; break; }
         if (sm < 0) break;
+        int64_t slot = 0;                        /* lowest free slot on that SM */
+        for (;; slot++) {
+          int used = 0;
+          for (k = 0; k < nres; k++)
+            if (sm_of[res[k]] == sm && slot_of[res[k]] == slot) used = 1;
+          if (!used) break;
+        }
         sm_of[c] = sm;
+        slot_of[c] = slot;
         if (cta_sm) cta_sm[c] = (int32_t)sm;
         res[nres++] = c;
         next_cta++;
         progress = 1;
       }
-      /* (2) issue the lowest-id issuable warp head */
+      /* (2) issue the lowest-id issuable warp head (per-subpartition
+       *     policies: the lowest id among the schedulers' picks) */
       int64_t best = -1;
+      for (k = 0; k < nq; k++) cand[k] = -1;
       for (k = 0; k < nres; k++) {
         const int64_t cc = res[k], sm = sm_of[cc];
         for (w = 0; w < W; w++) {
           const int64_t h = head[cc * W + w];
           if (h < 0 || npend[h] != 0 || rdy[h] > t) continue;
+          const int64_t l = slot_of[cc] * W + w, q = nsub ? sm * nsub + l % nsub : 0;
+          if (nsub && sub_avail[q] > t) continue; /* this scheduler already issued at t */
           if (cls[h] >= 0) {
             int ok = 0;
             for (int64_t q = 0; q < cap[cls[h]]; q++)
@@ -218,9 +257,21 @@ int oracle_simulate(
               if (hsrv[q] <= t) ok = 1;
             if (!ok) continue;
           }
-          if (best < 0 || h < best) best = h;
+          if (!nsub) {
+            if (best < 0 || h < best) best = h;
+            continue;
+          }
+          int64_t key;
+          if (policy == POL_GTO)
+            key = (l == sub_last[q] ? 0 : ((int64_t)1 << 40)) + cc * W + w;
+          else
+            key = sub_last[q] < 0 ? l : ((l - sub_last[q] - 1) % per + per) % per;
+          if (cand[q] < 0 || key < cand_key[q]) { cand[q] = h; cand_key[q] = key; }
         }
       }
+      if (nsub)
+        for (k = 0; k < nq; k++)
+          if (cand[k] >= 0 && (best < 0 || cand[k] < best)) best = cand[k];
       if (best >= 0) {
         v = best;
         c = cta[v];
@@ -229,6 +280,11 @@ int oracle_simulate(
         if (f > INT32_LIMIT) { status = OR_ERR_OVERFLOW; goto out; }
         start[v] = t;
         finish[v] = f;
+        if (nsub) {
+          const int64_t l = slot_of[c] * W + warp[v], q = sm * nsub + l % nsub;
+          sub_avail[q] = t + 1;
+          sub_last[q] = l;
+        }
         if (f > mkspan) mkspan = f;
         if (cls[v] >= 0) busy_acc[cls[v]] += occ[v];
         if (hocc[v] >= 0) busy_acc[RC_COUNT] += hocc[v];
@@ -271,6 +327,9 @@ int oracle_simulate(
         if (srv[r][k] > t && srv[r][k] < tn) tn = srv[r][k];
     for (k = 0; k < cap_hbm; k++)
       if (hsrv[k] > t && hsrv[k] < tn) tn = hsrv[k];
+    if (nsub)
+      for (k = 0; k < nq; k++)
+        if (sub_avail[k] > t && sub_avail[k] < tn) tn = sub_avail[k];
     if (tn == INT64_MAX) { status = OR_ERR_DEADLOCK; goto out; }
     t = tn;
   }
@@ -281,6 +340,7 @@ int oracle_simulate(
 out:
   free(cls); free(occ); free(hocc); free(lat); free(npend); free(rdy); free(nxt); free(head);
   free(rem); free(endt); free(sm_of); free(res); free(res_cnt); free(hsrv);
+  free(slot_of); free(sub_avail); free(sub_last); free(cand); free(cand_key);
   for (r = 0; r < RC_COUNT; r++) free(srv[r]);
   return status;
 }

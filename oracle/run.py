@@ -74,7 +74,7 @@ def simulate_arrays(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_
              work=np.ascontiguousarray(work, np.uint32), lat_extra=np.ascontiguousarray(lat_extra, np.uint32),
              cta_kernel=np.ascontiguousarray(cta_kernel, np.uint32))
     prm = np.ascontiguousarray(params, np.int32)
-    assert prm.shape == (24,)
+    assert prm.shape == (32,)
     n = a["type"].shape[0]
     m = a["col"].shape[0]
     C = a["cta_kernel"].shape[0]

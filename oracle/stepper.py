@@ -9,7 +9,10 @@ purpose in everything but the definition:
   CTA residency are recomputed from the partial schedule at every decision;
 * a resource class is free at t when fewer than ``cap`` of the nodes already
   started on it satisfy start <= t < start + occupancy (counting, not the
-  server free-time multiset the oracle keeps).
+  server free-time multiset the oracle keeps);
+* under the per-subpartition issue policies, a scheduler has issued at t when
+  a node of its warp slots started at t, and the slot it issued from last is
+  that of its latest-started node (read off the schedule, no scheduler state).
 
 Pure Python; only for graphs of a few dozen nodes with short latencies.
 """
@@ -52,6 +55,8 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     C = len(cta_kernel)
     prm = [int(x) for x in prm]
     num_sms, cps = prm[0], prm[1]
+    policy, nsub = prm[20], prm[21]
+    per = cps * warps_per_cta
     cap = {"tensor": prm[13], "tma": prm[14], "lsu": prm[15], "alu": prm[16], "bar": prm[17]}
     cap_hbm = prm[18]
     costs = [node_costs(int(type_[v]), int(work[v]), int(lat_extra[v]), prm) for v in range(n)]
@@ -62,10 +67,11 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     members = [[v for v in range(n) if int(cta[v]) == c] for c in range(C)]
     start = [None] * n
     cta_sm = [-1] * C
+    cta_slot = [-1] * C
     launched = [False] * C
     total_lat = sum(c[3] for c in costs)
-    if t_limit is None:
-        t_limit = total_lat + 2
+    if t_limit is None:   # every cycle without an issue lies under some node's latency or issue slot
+        t_limit = total_lat + n + 2
 
     def finish(v):
         return start[v] + costs[v][3]
@@ -89,6 +95,32 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     def busy_hbm(t):
         return sum(1 for u in range(n) if start[u] is not None and costs[u][2] is not None
                    and start[u] <= t < start[u] + costs[u][2])
+
+    def sched(v):
+        """(SM, scheduler, warp slot) of node v's warp."""
+        c = int(cta[v])
+        slot = cta_slot[c] * warps_per_cta + int(warp[v])
+        return cta_sm[c], slot % nsub, slot
+
+    def scheduler_picks(cands, t):
+        """Per scheduler that has not issued at t, its first candidate in policy order."""
+        groups = {}
+        for v in cands:
+            groups.setdefault(sched(v)[:2], []).append(v)
+        picks = []
+        for key, vs in groups.items():
+            mine = [u for u in range(n) if start[u] is not None and sched(u)[:2] == key]
+            if any(start[u] == t for u in mine):
+                continue
+            last = sched(max(mine, key=lambda u: start[u]))[2] if mine else None
+
+            def order(v):
+                slot = sched(v)[2]
+                if policy == 1:   # greedy-then-oldest
+                    return (slot != last, int(cta[v]) * warps_per_cta + int(warp[v]))
+                return slot if last is None else (slot - last - 1) % per   # round-robin
+            picks.append(min(vs, key=order))
+        return picks
 
     def issuable(v, t):
         c = int(cta[v])
@@ -129,8 +161,12 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
                     break
                 launched[c] = True
                 cta_sm[c] = free[0]
+                taken = {cta_slot[d] for d in range(c) if cta_sm[d] == free[0] and not retired(d, t)}
+                cta_slot[c] = min(k for k in range(cps) if k not in taken)
                 changed = True
             cands = [v for v in range(n) if issuable(v, t)]
+            if cands and nsub:
+                cands = scheduler_picks(cands, t)
             if cands:
                 v = min(cands)
                 start[v] = t

@@ -140,9 +140,13 @@ static_assert(SM_WORDS % 2 == 0, "SM records are read as 8-byte pairs");
 // CTA slot record (3 words): CTA id, nodes not issued, max finish
 constexpr uint32_t C_ID = 0, C_REM = 1, C_END = 2, CTA_WORDS = 3;
 
+// Scheduler record (2 words, per-subpartition policies only): first cycle it
+// may issue again, warp slot on the SM it issued from last (NONE: never)
+constexpr uint32_t Q_AVAIL = 0, Q_LAST = 1, SUB_WORDS = 2;
+
 struct Layout {
-  uint32_t S, Scta, NS, SC, cap_hbm, per;
-  uint32_t o_slot, o_sm, o_cta, o_sv, o_hs, words;
+  uint32_t S, Scta, NS, SC, cap_hbm, per, nsub;
+  uint32_t o_slot, o_sm, o_cta, o_sv, o_hs, o_sub, words;
 };
 
 __host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
@@ -155,7 +159,15 @@ __host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
   for (int i = GTS_P_CAP_TENSOR; i <= GTS_P_CAP_HBM; i++)
     if (p[i] < 1) return GTS_ERR_INVALID_PARAMS;
   if (p[GTS_P_GRAPH_INDEX] < 0 || (uint32_t)p[GTS_P_GRAPH_INDEX] >= G) return GTS_ERR_INVALID_PARAMS;
-  for (int i = 20; i < GTS_NPARAM; i++)
+  const int32_t pol = p[GTS_P_ISSUE_POLICY], nsub = p[GTS_P_SUBPARTITIONS];
+  if (pol == GTS_POLICY_LOWEST_ID) {
+    if (nsub != 0) return GTS_ERR_INVALID_PARAMS;
+  } else if (pol == GTS_POLICY_GTO || pol == GTS_POLICY_RR) {
+    if (nsub < 1 || nsub > 32) return GTS_ERR_INVALID_PARAMS;
+  } else {
+    return GTS_ERR_INVALID_PARAMS;
+  }
+  for (int i = GTS_P_SUBPARTITIONS + 1; i < GTS_NPARAM; i++)
     if (p[i] != 0) return GTS_ERR_INVALID_PARAMS;
   return GTS_OK;
 }
@@ -190,6 +202,8 @@ __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint3
   L.o_cta = (uint32_t)w; w += (uint64_t)L.Scta * CTA_WORDS;
   L.o_sv = (uint32_t)w; w += (uint64_t)L.NS * L.SC;
   L.o_hs = (uint32_t)w; w += L.cap_hbm;
+  L.nsub = (uint32_t)p[GTS_P_SUBPARTITIONS];
+  L.o_sub = (uint32_t)w; w += (uint64_t)L.NS * L.nsub * SUB_WORDS;
   w = (w + 3) & ~(uint64_t)3;  // 16-byte multiple
   if (w * 4 > MAX_SMEM_BYTES) return false;
   L.words = (uint32_t)w;
@@ -238,11 +252,15 @@ struct Pt {
   uint2 *scr;        // scratch counters (graph-local index)
   uint64_t offs;     // byte r: offset of class r's servers inside an SM's servers
   uint32_t caps;     // 6 bits per class: servers of class r (0: class unused)
+  uint32_t policy;   // GTS_POLICY_*; L.nsub > 0 for the per-subpartition policies
   __device__ __forceinline__ uint32_t cls_off(uint32_t r) const { return (uint32_t)(offs >> (8 * r)) & 255u; }
   __device__ __forceinline__ uint32_t cls_cap(uint32_t r) const { return (caps >> (6 * r)) & 63u; }
   __device__ __forceinline__ uint32_t *slot(uint32_t i) const { return sp + L.o_slot + i * SLOT_WORDS; }
   __device__ __forceinline__ uint32_t *smrec(uint32_t s) const { return sp + L.o_sm + s * SM_WORDS; }
   __device__ __forceinline__ uint32_t *cta(uint32_t j) const { return sp + L.o_cta + j * CTA_WORDS; }
+  __device__ __forceinline__ uint32_t *sub(uint32_t s, uint32_t u) const {
+    return sp + L.o_sub + (s * L.nsub + u) * SUB_WORDS;
+  }
 };
 
 // Occupancies and latency of a node (Section 5.2 throughput model).
@@ -275,9 +293,68 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
   return k;
 }
 
+// One lane: SM s's record under per-subpartition schedulers (Section 5.3,
+// greedy-then-oldest / round-robin).  Scheduler u's event is
+// E_u = max(first cycle it may issue, least effective key of its heads); its
+// pick is the first head in policy order among those whose effective key is
+// <= E_u.  The record holds the least (E_u, id of the pick) over u.
+__device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
+  const uint32_t per = P.L.per, nsub = P.L.nsub, i0 = s * per;
+  const uint32_t nl = min(per, P.L.S - i0);
+  uint64_t best = INF64;
+  uint32_t bsl = 0, hmin = INF;
+  for (uint32_t u = 0; u < nsub; u++) {
+    const uint32_t *sq = P.sub(s, u);
+    uint32_t m = INF;
+    for (uint32_t l = u; l < nl; l += nsub) {
+      const uint32_t k = slot_key(P, i0 + l, t);
+      if (k == INF) continue;
+      if (P.slot(i0 + l)[F_HID] & HBM_BIT) {
+        hmin = min(hmin, k);
+        m = min(m, max(k, H));
+      } else {
+        m = min(m, k);
+      }
+    }
+    if (m == INF) continue;
+    const uint32_t E = max(m, sq[Q_AVAIL]), last = sq[Q_LAST];
+    uint64_t bp = INF64;  // (policy key << 32 | slot)
+    for (uint32_t l = u; l < nl; l += nsub) {
+      const uint32_t k = slot_key(P, i0 + l, t);
+      if (k == INF) continue;
+      const uint32_t e = (P.slot(i0 + l)[F_HID] & HBM_BIT) ? max(k, H) : k;
+      if (e > E) continue;
+      uint32_t key;
+      if (P.policy == GTS_POLICY_GTO) {  // greedy slot, then the oldest warp (CTA id, warp)
+        key = (l == last ? 0u : 0x80000000u) | (P.cta((i0 + l) / P.W)[C_ID] * P.W + l % P.W);
+      } else {                            // round-robin after the last slot
+        key = last == NONE ? l : (l + per - last - 1u) % per;
+      }
+      bp = min(bp, pack(key, l));
+    }
+    const uint32_t lc = (uint32_t)bp;
+    const uint64_t val = pack(E, P.slot(i0 + lc)[F_HID] & ID_MASK);
+    if (val < best) {
+      best = val;
+      bsl = i0 + lc;
+    }
+  }
+  uint32_t *o = P.smrec(s);
+  o[0] = (uint32_t)best;
+  o[1] = (uint32_t)(best >> 32);
+  o[2] = bsl;
+  o[3] = hmin;
+}
+
 // Warp-parallel: the keys of SM s's heads at cycle t and the SM's summary
 // record.  All lanes call it.
+template <bool SCHED>
 __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane) {
+  if (SCHED && P.L.nsub) {
+    if (lane == 0) rescan_sm_sub(P, s, t, H);
+    __syncwarp();
+    return;
+  }
   const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
   uint64_t best = INF64;
   uint32_t bsl = 0, hmin = INF;
@@ -312,7 +389,12 @@ __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, 
 }
 
 // One lane: recompute the record of SM s at cycle t and horizon H.
+template <bool SCHED>
 __device__ __forceinline__ void rescan_sm_lane(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
+  if (SCHED && P.L.nsub) {
+    rescan_sm_sub(P, s, t, H);
+    return;
+  }
   const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
   uint64_t best = INF64;
   uint32_t bsl = 0, hmin = INF;
@@ -395,6 +477,7 @@ struct Clock {
 
 // Retire finished CTAs and launch as many CTAs as fit at cycle t (Section 5.1
 // TB scheduler; kernel-boundary gate).  Returns false on step-limit.
+template <bool SCHED>
 __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_row, int lane, uint64_t &b,
                             uint32_t &bsl) {
   const uint32_t t = C.t;
@@ -451,12 +534,15 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
     }
     __syncwarp();
     const uint32_t s = freeslot / P.cps;
-    refresh_sm(P, s, t, C.H, lane);
+    refresh_sm<SCHED>(P, s, t, C.H, lane);
     refresh_owner(P, s & 31u, lane, b, bsl);
     C.next_cta++;
   }
 }
 
+// SCHED: the kernel instance that also runs the per-subpartition issue
+// policies; the host launches the plain instance when no row asks for them.
+template <bool SCHED>
 __global__ void __launch_bounds__(MAX_WPB * 32, 1)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
@@ -486,7 +572,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     P.c1 = g.cta_off[gi + 1];
     const uint32_t CG = P.c1 - P.c0;
     if (status == GTS_OK) {
-      if (!make_layout(prm, CG, P.W, g.class_mask, P.L) || P.L.words > budget_words) status = GTS_ERR_UNSUPPORTED;
+      if (!make_layout(prm, CG, P.W, g.class_mask, P.L) || P.L.words > budget_words || (!SCHED && P.L.nsub))
+        status = GTS_ERR_UNSUPPORTED;
     }
     if (status != GTS_OK) {
       if (lane == 0) {
@@ -499,6 +586,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       continue;
     }
     P.cps = (uint32_t)prm[GTS_P_CTAS_PER_SM];
+    P.policy = (uint32_t)prm[GTS_P_ISSUE_POLICY];
     P.st = (flags & GTS_FULL_TRACE) ? d_start + (size_t)q * g.row_nodes : nullptr;
     P.fi = (flags & GTS_FULL_TRACE) ? d_finish + (size_t)q * g.row_nodes : nullptr;
     P.scr = scratch + (size_t)gw * ((g.row_nodes + 1u) & ~1u);
@@ -544,6 +632,10 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     for (uint32_t j = lane; j < P.L.Scta; j += 32) P.cta(j)[C_ID] = NONE;
     for (uint32_t k = lane; k < P.L.NS * P.L.SC; k += 32) sp[P.L.o_sv + k] = 0u;
     for (uint32_t k = lane; k < P.L.cap_hbm; k += 32) sp[P.L.o_hs + k] = 0u;
+    for (uint32_t k = lane; k < P.L.NS * P.L.nsub; k += 32) {
+      sp[P.L.o_sub + k * SUB_WORDS + Q_AVAIL] = 0u;
+      sp[P.L.o_sub + k * SUB_WORDS + Q_LAST] = NONE;
+    }
     {
       uint4 *z = reinterpret_cast<uint4 *>(P.scr);
       const uint32_t nz = nG / 2;
@@ -568,7 +660,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     uint64_t busy = 0;  // lane r < 5: server-cycles of per-SM class r; lane 5: HBM
     uint64_t b = INF64;  // this lane's best (effective cycle << 32 | id) over its SMs
     uint32_t bsl = 0;    // ... and its slot
-    if (!launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
+    if (!launch_ctas<SCHED>(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
 
     while (status == GTS_OK && issued < nG) {
       // ---- next event: minimum of (effective cycle, node id) over all heads
@@ -581,7 +673,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
         C.t = tn;
         if (C.next_ret <= C.t) {  // a CTA retires first: launch, then choose again
-          if (!launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
+          if (!launch_ctas<SCHED>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
           continue;
         }
         // otherwise the minimum just found is the first issue at the new cycle
@@ -625,6 +717,12 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         const bool fr = (uint32_t)lane < P.cls_cap(cls) && sv[lane] <= t;
         const uint32_t bal = __ballot_sync(FULL, fr);
         if (lane == __ffs(bal) - 1) sv[lane] = t + occ;
+      }
+      if (SCHED && P.L.nsub && lane == 0) {  // the issuing scheduler: one issue per cycle, remember the slot
+        const uint32_t l = i - sm * P.L.per;
+        uint32_t *sq = P.sub(sm, l % P.L.nsub);
+        sq[Q_AVAIL] = t + 1u;
+        sq[Q_LAST] = l;
       }
       // take one free global HBM server
       const uint32_t prevH = C.H;
@@ -705,17 +803,17 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
       if (cross_touch) {  // a release reached a head of another CTA: recompute everything
-        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane(P, s, t, C.H);
+        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane<SCHED>(P, s, t, C.H);
         __syncwarp();
         b = lane_best(P, lane, bsl);
       } else {
-        refresh_sm(P, sm, t, C.H, lane);
+        refresh_sm<SCHED>(P, sm, t, C.H, lane);
         if (C.H != prevH) {
           // SMs whose HBM heads H overtakes change their effective cycles
           bool any = false;
           for (uint32_t s = lane; s < P.L.NS; s += 32) {
             if (s != sm && P.smrec(s)[3] < C.H) {
-              rescan_sm_lane(P, s, t, C.H);
+              rescan_sm_lane<SCHED>(P, s, t, C.H);
               any = true;
             }
           }
@@ -727,7 +825,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       __syncwarp();
       if (rem == 0u) {
         if (cend <= t) {
-          if (!launch_ctas(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
+          if (!launch_ctas<SCHED>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
         } else {
           C.next_ret = min(C.next_ret, cend);
         }
@@ -785,6 +883,7 @@ struct gts_params {
   const int32_t *d_params;
   uint32_t n_points;
   std::vector<uint32_t> words;  // per row: shared words, 0 if the row is invalid or too large
+  std::vector<uint8_t> sched;   // per row: asks for a per-subpartition issue policy
 };
 
 struct gts_results {
@@ -961,9 +1060,11 @@ gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_p
   P->d_params = d_params;
   P->n_points = n_points;
   P->words.assign(n_points, 0u);
+  P->sched.assign(n_points, 0u);
   for (uint32_t p = 0; p < n_points; p++) {
     const int32_t *row = h.data() + (size_t)p * GTS_NPARAM;
     if (check_row(row, g->G) != GTS_OK) continue;
+    P->sched[p] = row[GTS_P_ISSUE_POLICY] != GTS_POLICY_LOWEST_ID;
     const uint32_t gi = (uint32_t)row[GTS_P_GRAPH_INDEX];
     Layout L;
     if (make_layout(row, g->cta_off[gi + 1] - g->cta_off[gi], g->W, g->dg.class_mask, L)) P->words[p] = L.words;
@@ -984,17 +1085,23 @@ uint64_t scratch_row_bytes(const gts_graph *g) { return (((uint64_t)g->dg.row_no
 
 struct Plan {
   uint32_t words, wpb, smem, blocks, warps;
+  bool sched;  // launch the instance with the per-subpartition policies
 };
 
 gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, uint32_t np, uint32_t flags,
                        size_t scratch_bytes, bool limit_by_scratch, Plan &pl) {
   (void)flags;
   uint32_t words = 64;
-  for (uint32_t p = first; p < first + np; p++) words = std::max(words, P->words[p]);
+  pl.sched = false;
+  for (uint32_t p = first; p < first + np; p++) {
+    words = std::max(words, P->words[p]);
+    pl.sched = pl.sched || P->sched[p];
+  }
   const uint32_t bytes = words * 4;
   pl.words = words;
-  cudaError_t e = cudaFuncSetAttribute(k_simulate, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)MAX_SMEM_BYTES);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_simulate, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  const void *kern = pl.sched ? (const void *)k_simulate<true> : (const void *)k_simulate<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)MAX_SMEM_BYTES);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -1005,7 +1112,7 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
   for (uint32_t wpb = MAX_WPB; wpb >= 1; wpb--) {
     if (wpb * bytes > MAX_SMEM_BYTES) continue;
     int nb = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_simulate, (int)wpb * 32, wpb * bytes);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kern, (int)wpb * 32, wpb * bytes);
     if (e != cudaSuccess) return cuda_fail(e, "simulate: occupancy query");
     if ((uint32_t)nb * wpb > best_w) {
       best_w = (uint32_t)nb * wpb;
@@ -1060,7 +1167,8 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
     Plan pl;
     gts_status st = plan_launch(g, P, first_point, n_points, flags, scratch_bytes, true, pl);
     if (st != GTS_OK) return st;
-    k_simulate<<<pl.blocks, pl.wpb * 32, pl.smem, s>>>(
+    auto kern = pl.sched ? k_simulate<true> : k_simulate<false>;
+    kern<<<pl.blocks, pl.wpb * 32, pl.smem, s>>>(
         g->dg, P->d_params, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status,
         (flags & GTS_WANT_DIGEST) ? d_digest : nullptr, (flags & GTS_WANT_CTA_SM) ? d_cta_sm : nullptr,
         (flags & GTS_WANT_BUSY) ? d_busy : nullptr, (uint2 *)d_scratch, pl.warps, pl.words);

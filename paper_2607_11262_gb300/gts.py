@@ -38,6 +38,9 @@ GTS_BUSY_CLASSES = 6
 GTS_BUSY_TENSOR, GTS_BUSY_TMA, GTS_BUSY_LSU, GTS_BUSY_ALU, GTS_BUSY_BAR, GTS_BUSY_HBM = range(6)
 BUSY_NAMES = ("tensor", "tma", "lsu", "alu", "bar", "hbm")
 
+GTS_NPARAM = 32
+GTS_POLICY_LOWEST_ID, GTS_POLICY_GTO, GTS_POLICY_RR = 0, 1, 2
+
 GTS_STATIC_SCRATCH_BYTES = 32 << 20
 
 EXPORTS = ("gts_graph_workspace_bytes", "gts_graph_create", "gts_graph_destroy", "gts_params_upload",
@@ -249,13 +252,15 @@ class DeviceGraph:
 
 
 class DeviceParams:
-    """A [P][24] int32 parameter table resident on the GPU."""
+    """A [P][GTS_NPARAM] int32 parameter table resident on the GPU."""
 
     def __init__(self, dgraph: DeviceGraph, params, stream=None, tensor=None, n_points=None):
         import torch
         self.dgraph = dgraph
         if tensor is None:
             p = np.ascontiguousarray(params, np.int32)
+            if p.ndim != 2 or p.shape[1] != GTS_NPARAM:
+                raise ValueError(f"params must be [n_points][{GTS_NPARAM}] int32, got {p.shape}")
             self.n_points = int(p.shape[0])
             self.tensor = torch.from_numpy(p.reshape(-1)).to(dgraph.workspace.device)
         else:

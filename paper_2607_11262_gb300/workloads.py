@@ -37,16 +37,19 @@ LOAD, SMEM, MMA, EW, STORE, BAR, NOP = range(7)
 TYPE_NAMES = ("LOAD", "SMEM", "MMA", "EW", "STORE", "BAR", "NOP")
 DATA, ISSUE = 0, 1
 
-NPARAM = 24
+NPARAM = 32
 (P_NUM_SMS, P_CTAS_PER_SM, P_HBM_BPC, P_DRAM_LAT, P_TMA_BPC, P_TMA_LAT,
  P_SMEM_BPC, P_SMEM_LAT, P_MMA_FMA_PC, P_MMA_LAT, P_ALU_OPS_PC, P_ALU_LAT,
  P_BAR_LAT, P_CAP_TENSOR, P_CAP_TMA, P_CAP_LSU, P_CAP_ALU, P_CAP_BAR,
- P_CAP_HBM, P_GRAPH_INDEX) = range(20)
+ P_CAP_HBM, P_GRAPH_INDEX, P_ISSUE_POLICY, P_SUBPARTITIONS) = range(22)
 PARAM_NAMES = ("num_sms", "ctas_per_sm", "hbm_bpc", "dram_lat", "tma_bpc",
                "tma_lat", "smem_bpc", "smem_lat", "mma_fma_pc", "mma_lat",
                "alu_ops_pc", "alu_lat", "bar_lat", "cap_tensor", "cap_tma",
                "cap_lsu", "cap_alu", "cap_bar", "cap_hbm", "graph_index",
-               "reserved20", "reserved21", "reserved22", "reserved23")
+               "issue_policy", "subpartitions") + tuple(f"reserved{i}" for i in range(22, NPARAM))
+# issue policies (Section 5.3): one global lowest-id order, or per-subpartition
+# greedy-then-oldest / round-robin schedulers issuing one node per cycle
+POLICY_LOWEST_ID, POLICY_GTO, POLICY_RR = 0, 1, 2
 
 H100_CORE_HZ = 1.98e9  # H100 SXM core clock, Table "GPU configurations"
 

@@ -9,6 +9,8 @@
   makespan; finish = start + latency; no unit over capacity at any cycle; warp
   starts are non-decreasing; Graham's (2 - 1/m) bound against a brute-force
   optimum of P|prec|Cmax;
+* per-subpartition issue policies (greedy-then-oldest, round-robin): hand
+  schedules, stepper == oracle, one issue per scheduler per cycle;
 * busy server-cycles: equal to the stepper's cycle-by-cycle count of held
   servers; a single saturated server is busy for the whole makespan; busy
   cycles never exceed servers x makespan;
@@ -77,6 +79,81 @@ def test_golden_hand_schedules():
         assert r.makespan == case["makespan"], case["name"]
         assert list(r.cta_sm) == case["cta_sm"], case["name"]
         assert_same(r, s)
+
+
+def test_golden_issue_policies():
+    spec = json.load(open(os.path.join(GOLDEN, "issue_policies.json")))
+    for case in spec["cases"]:
+        nodes = case["nodes"]
+        g = TG.make(len(nodes), [(u, v, KIND[k]) for u, v, k in case["edges"]],
+                    [TYPE[x[0]] for x in nodes], [x[1] for x in nodes], [x[2] for x in nodes],
+                    case["warps_per_cta"], work=[x[3] for x in nodes])
+        prm = TG.unit_params(case["num_sms"], case["ctas_per_sm"])
+        prm[W.P_ISSUE_POLICY] = case["policy"]
+        prm[W.P_SUBPARTITIONS] = case["subpartitions"]
+        r, s = both(g, prm)
+        assert r.status == 0, case["name"]
+        assert list(r.start) == case["start"], (case["name"], list(r.start))
+        assert_same(r, s)
+
+
+def _with_policy(prm, policy, nsub):
+    prm = prm.copy()
+    prm[W.P_ISSUE_POLICY] = policy
+    prm[W.P_SUBPARTITIONS] = nsub
+    return prm
+
+
+@pytest.mark.parametrize("policy", [W.POLICY_GTO, W.POLICY_RR])
+def test_stepper_equals_oracle_policies(policy):
+    rng = np.random.default_rng(40 + policy)
+    for n in (1, 2, 3):
+        for edges in TG.all_edge_sets(n):
+            types = [int(x) for x in rng.integers(0, 7, n)]
+            warps = [int(x) for x in rng.integers(0, 3, n)]
+            ctas = sorted(int(x) for x in rng.integers(0, 2, n))
+            g = TG.make(n, edges, types, warps, ctas, 3, work=[int(x) for x in rng.integers(0, 4, n)])
+            prm = _with_policy(TG.small_params(rng, 1, 2), policy, int(rng.integers(1, 4)))
+            r, s = both(g, prm)
+            assert_same(r, s)
+    for i in range(120):
+        n = int(rng.integers(5, 22))
+        g = TG.random_graph(rng, n, p_edge=float(rng.uniform(0.05, 0.35)), cta_major=bool(i % 3),
+                            kernels=bool(i % 2))
+        prm = _with_policy(TG.small_params(rng), policy, int(rng.integers(1, 5)))
+        r, s = both(g, prm)
+        assert_same(r, s)
+
+
+@pytest.mark.parametrize("policy", [W.POLICY_GTO, W.POLICY_RR])
+def test_one_issue_per_scheduler_per_cycle(policy):
+    # W independent zero-latency warps of k nodes on one scheduler: the n nodes
+    # start at 0, 1, ..., n-1 (no idle cycle, never two in one cycle); with s
+    # schedulers every cycle issues min(s, warps left) nodes
+    rng = np.random.default_rng(50 + policy)
+    for _ in range(20):
+        Wn = int(rng.integers(1, 6))
+        k = int(rng.integers(1, 5))
+        n = Wn * k
+        g = TG.make(n, [], [W.NOP] * n, [v % Wn for v in range(n)], [0] * n, Wn, work=[0] * n)
+        r = run.simulate(g, _with_policy(TG.unit_params(1, 1), policy, 1))
+        assert r.status == 0
+        assert sorted(r.start) == list(range(n))
+        if Wn > 1:
+            r2 = run.simulate(g, _with_policy(TG.unit_params(1, 1), policy, Wn))
+            assert list(r2.start) == [v // Wn for v in range(n)]
+
+
+def test_policy_parameter_checks():
+    g = TG.make(2, [], [W.NOP, W.NOP], [0, 1], [0, 0], 2, work=[0, 0])
+    base = TG.unit_params(1, 1)
+    for policy, nsub in ((0, 1), (1, 0), (2, 33), (3, 1), (-1, 0)):
+        assert run.simulate(g, _with_policy(base, policy, nsub)).status == run.ERR_INVALID_PARAMS
+    bad = base.copy()
+    bad[W.NPARAM - 1] = 1          # reserved
+    assert run.simulate(g, bad).status == run.ERR_INVALID_PARAMS
+    for policy, nsub in ((0, 0), (1, 1), (2, 32)):
+        assert run.simulate(g, _with_policy(base, policy, nsub)).status == 0
 
 
 # ------------------------------------------------------------------ brute force
