@@ -73,6 +73,9 @@ typedef int32_t gts_status;
 #define GTS_STORE 4   /* shared/registers -> global; work = bytes; TMA + HBM; base tma_lat */
 #define GTS_BAR   5   /* mbarrier / named-barrier wait; BAR for 1 cycle; base bar_lat */
 #define GTS_NOP   6   /* pure synchronisation point; no unit; base 0 */
+#define GTS_DSMEM 7   /* remote shared-memory access inside an SM group (DSMEM, Section 5.2 "DSMEM / On-chip
+                         NoC"); work = bytes; LSU on its own SM + one NoC server of its SM group;
+                         base smem_lat + noc_lat */
 
 /* Edge kinds (Section 4.1 data and order edges). */
 #define GTS_EDGE_DATA  0  /* released when the producer completes */
@@ -103,7 +106,13 @@ typedef int32_t gts_status;
 #define GTS_P_GRAPH_INDEX 19   /* which graph of a stacked set this point runs */
 #define GTS_P_ISSUE_POLICY 20  /* GTS_POLICY_*, see below */
 #define GTS_P_SUBPARTITIONS 21 /* issue schedulers per SM: 1..32 for GTO / RR, 0 for LOWEST_ID */
-/* 22..31 reserved, must be 0 */
+#define GTS_P_NOC_BPC      22  /* on-chip NoC bytes per cycle per NoC server */
+#define GTS_P_NOC_LAT      23  /* NoC latency added to a DSMEM node's base */
+#define GTS_P_CAP_NOC      24  /* NoC servers per SM group (1..32) */
+#define GTS_P_CLUSTER_SMS  25  /* SMs per NoC group: SM s is in group s / cluster_sms (1..32) */
+/* NoC fields 22..25 are all 0 (no NoC: a graph with DSMEM nodes is then GTS_ERR_INVALID_PARAMS
+ * for that row) or noc_bpc >= 1, noc_lat >= 0, 1 <= cap_noc <= 32, 1 <= cluster_sms <= 32.
+ * 26..31 reserved, must be 0 */
 
 /*
  * Issue policies (Section 5.3: ready nodes sit in per-subpartition queues
@@ -138,14 +147,16 @@ typedef int32_t gts_status;
  * r of occ_r(v), the cycles v holds one server of r.  Class r's utilisation
  * over the run (Section 7.1 reports it for the tensor cores) is
  * busy_r / (servers_r * makespan), with servers_r = cap_r * num_sms for the
- * per-SM classes and cap_hbm for HBM. */
-#define GTS_BUSY_CLASSES 6
+ * per-SM classes, cap_hbm for HBM and cap_noc * ceil(num_sms / cluster_sms)
+ * for the NoC. */
+#define GTS_BUSY_CLASSES 7
 #define GTS_BUSY_TENSOR  0
 #define GTS_BUSY_TMA     1
 #define GTS_BUSY_LSU     2
 #define GTS_BUSY_ALU     3
 #define GTS_BUSY_BAR     4
 #define GTS_BUSY_HBM     5
+#define GTS_BUSY_NOC     6
 
 typedef struct gts_graph gts_graph;
 typedef struct gts_params gts_params;
@@ -160,7 +171,7 @@ typedef struct gts_results gts_results;
  *    row_ptr[n_nodes] = n_edges; col[e] is the successor, ekind[e] its kind;
  *  - every edge u->v has u < v and stays inside its graph (ids are a
  *    topological order);
- *  - type < 7, warp < warps_per_cta, cta inside the node's graph;
+ *  - type < 8, warp < warps_per_cta, cta inside the node's graph;
  *  - cta_kernel is non-decreasing within each graph.
  * The program order of each (cta, warp) stream is ascending id.
  * Limits: n_nodes < 2^31, n_ctas < 2^24, warps_per_cta <= 128, in-degree

@@ -18,7 +18,9 @@
  *     type ty takes one server of each resource class it uses for its
  *     occupancy occ = ceil(work / rate) cycles; its latency is
  *     L = base(ty) + lat_extra + max over used classes of occ.  Per-SM classes:
- *     TENSOR, TMA, LSU, ALU, BAR; one global class: HBM.
+ *     TENSOR, TMA, LSU, ALU, BAR; one global class: HBM; one class per group
+ *     of cluster_sms consecutive SMs: the on-chip NoC that DSMEM nodes (remote
+ *     shared-memory accesses, Section 5.2 "DSMEM / On-chip NoC") cross.
  *   - Thread blocks are bound to SMs in ascending CTA order, each to the lowest
  *     SM with a free slot; a CTA retires when all its nodes completed and then
  *     frees its slot (Section 5.1).  A CTA of kernel k launches only after
@@ -63,7 +65,8 @@
 #define OR_ERR_DEADLOCK (-8)
 
 /* operation types (Section 4.1 operation descriptor) */
-enum { OT_LOAD = 0, OT_SMEM = 1, OT_MMA = 2, OT_EW = 3, OT_STORE = 4, OT_BAR = 5, OT_NOP = 6, OT_COUNT = 7 };
+enum { OT_LOAD = 0, OT_SMEM = 1, OT_MMA = 2, OT_EW = 3, OT_STORE = 4, OT_BAR = 5, OT_NOP = 6, OT_DSMEM = 7,
+       OT_COUNT = 8 };
 /* per-SM resource classes (Section 5.2) */
 enum { RC_TENSOR = 0, RC_TMA = 1, RC_LSU = 2, RC_ALU = 3, RC_BAR = 4, RC_COUNT = 5 };
 
@@ -72,7 +75,8 @@ enum {
   PR_NUM_SMS = 0, PR_CTAS_PER_SM, PR_HBM_BPC, PR_DRAM_LAT, PR_TMA_BPC, PR_TMA_LAT,
   PR_SMEM_BPC, PR_SMEM_LAT, PR_MMA_FMA_PC, PR_MMA_LAT, PR_ALU_OPS_PC, PR_ALU_LAT,
   PR_BAR_LAT, PR_CAP_TENSOR, PR_CAP_TMA, PR_CAP_LSU, PR_CAP_ALU, PR_CAP_BAR,
-  PR_CAP_HBM, PR_GRAPH_INDEX, PR_ISSUE_POLICY, PR_SUBPARTITIONS, PR_COUNT = 32
+  PR_CAP_HBM, PR_GRAPH_INDEX, PR_ISSUE_POLICY, PR_SUBPARTITIONS, PR_NOC_BPC, PR_NOC_LAT, PR_CAP_NOC,
+  PR_CLUSTER_SMS, PR_COUNT = 32
 };
 enum { POL_LOWEST_ID = 0, POL_GTO = 1, POL_RR = 2 };
 
@@ -87,14 +91,14 @@ int oracle_simulate(
     const uint32_t *work, const uint32_t *lat_extra, const uint32_t *cta_kernel,
     const int32_t *prm,
     int64_t *start, int64_t *finish, int64_t *makespan, int32_t *cta_sm,
-    int64_t *busy /* [RC_COUNT + 1]: per-SM classes, then HBM; may be NULL */)
+    int64_t *busy /* [RC_COUNT + 2]: per-SM classes, HBM, NoC; may be NULL */)
 {
   int64_t v, e, c, w, k, r;
   int status = OR_OK;
   if (n < 0 || m < 0 || n_ctas < 0 || W < 1 || !prm || !makespan) return OR_ERR_INVALID_ARG;
-  int64_t busy_acc[RC_COUNT + 1] = {0, 0, 0, 0, 0, 0};
+  int64_t busy_acc[RC_COUNT + 2] = {0, 0, 0, 0, 0, 0, 0};
   if (busy)
-    for (r = 0; r <= RC_COUNT; r++) busy[r] = 0;
+    for (r = 0; r < RC_COUNT + 2; r++) busy[r] = 0;
 
   /* ---- parameter row (Table "GPU configurations" quantities) ---- */
   const int64_t num_sms = prm[PR_NUM_SMS], cps = prm[PR_CTAS_PER_SM];
@@ -115,8 +119,17 @@ int oracle_simulate(
   } else {
     return OR_ERR_INVALID_PARAMS;
   }
-  for (k = PR_SUBPARTITIONS + 1; k < PR_COUNT; k++)
+  const int64_t noc_bpc = prm[PR_NOC_BPC], cap_noc = prm[PR_CAP_NOC], csms = prm[PR_CLUSTER_SMS];
+  const int noc = csms != 0;                 /* the row configures an on-chip NoC */
+  if (noc) {
+    if (noc_bpc < 1 || prm[PR_NOC_LAT] < 0 || cap_noc < 1 || cap_noc > 32 || csms < 1 || csms > 32)
+      return OR_ERR_INVALID_PARAMS;
+  } else if (noc_bpc != 0 || prm[PR_NOC_LAT] != 0 || cap_noc != 0) {
+    return OR_ERR_INVALID_PARAMS;
+  }
+  for (k = PR_CLUSTER_SMS + 1; k < PR_COUNT; k++)
     if (prm[k] != 0) return OR_ERR_INVALID_PARAMS;
+  const int64_t ngrp = noc ? (num_sms + csms - 1) / csms : 1;  /* NoC groups */
   const int64_t per = cps * W;               /* warp slots per SM */
   const int64_t nq = num_sms * (nsub ? nsub : 1);
 
@@ -130,6 +143,8 @@ int oracle_simulate(
   }
   for (c = 1; c < n_ctas; c++)
     if (cta_kernel[c] < cta_kernel[c - 1]) return OR_ERR_INVALID_GRAPH;
+  for (v = 0; v < n; v++)
+    if (type[v] == OT_DSMEM && !noc) return OR_ERR_INVALID_PARAMS;  /* the row has no NoC to serve it */
 
   /* ---- per-node occupancy and latency (Section 5.2, Section 5.3) ---- */
   int8_t *cls = malloc((size_t)(n ? n : 1));
@@ -152,9 +167,12 @@ int oracle_simulate(
   int64_t *cand_key = malloc(sizeof(int64_t) * (size_t)nq);
   int64_t *srv[RC_COUNT];
   int64_t *hsrv = calloc((size_t)cap_hbm, sizeof(int64_t));
+  int64_t *nsrv = calloc((size_t)(ngrp * (noc ? cap_noc : 1)), sizeof(int64_t)); /* NoC servers per group */
+  int64_t *nocc = malloc(sizeof(int64_t) * (size_t)(n ? n : 1));
   for (r = 0; r < RC_COUNT; r++) srv[r] = calloc((size_t)(num_sms * cap[r]), sizeof(int64_t));
   int nomem = !cls || !occ || !hocc || !lat || !npend || !rdy || !nxt || !head || !rem || !endt ||
-              !sm_of || !res || !res_cnt || !hsrv || !slot_of || !sub_avail || !sub_last || !cand || !cand_key;
+              !sm_of || !res || !res_cnt || !hsrv || !slot_of || !sub_avail || !sub_last || !cand || !cand_key ||
+              !nsrv || !nocc;
   for (r = 0; r < RC_COUNT; r++) nomem |= !srv[r];
   if (nomem) { status = OR_ERR_NOMEM; goto out; }
 
@@ -164,6 +182,7 @@ int oracle_simulate(
     cls[v] = -1;
     occ[v] = 0;
     hocc[v] = -1; /* -1: does not use HBM */
+    nocc[v] = -1; /* -1: does not cross the NoC */
     switch (type[v]) {
       case OT_LOAD:  cls[v] = RC_TMA; occ[v] = cdiv(wk, rate[RC_TMA]); hocc[v] = cdiv(wk, hbm_bpc);
                      base = prm[PR_TMA_LAT] + prm[PR_DRAM_LAT]; break;
@@ -173,10 +192,13 @@ int oracle_simulate(
       case OT_STORE: cls[v] = RC_TMA; occ[v] = cdiv(wk, rate[RC_TMA]); hocc[v] = cdiv(wk, hbm_bpc);
                      base = prm[PR_TMA_LAT]; break;
       case OT_BAR:   cls[v] = RC_BAR; occ[v] = 1; base = prm[PR_BAR_LAT]; break;
+      case OT_DSMEM: cls[v] = RC_LSU; occ[v] = cdiv(wk, rate[RC_LSU]); nocc[v] = cdiv(wk, noc_bpc);
+                     base = prm[PR_SMEM_LAT] + prm[PR_NOC_LAT]; break;
       default:       break; /* NOP: no resource, base 0 */
     }
     if (cls[v] >= 0 && occ[v] > mx) mx = occ[v];
     if (hocc[v] > mx) mx = hocc[v];
+    if (nocc[v] > mx) mx = nocc[v];
     lat[v] = base + (int64_t)lat_extra[v] + mx;
   }
 
@@ -257,6 +279,12 @@ int oracle_simulate(
               if (hsrv[q] <= t) ok = 1;
             if (!ok) continue;
           }
+          if (nocc[h] >= 0) {
+            int ok = 0;
+            for (int64_t q = 0; q < cap_noc; q++)
+              if (nsrv[(sm / csms) * cap_noc + q] <= t) ok = 1;
+            if (!ok) continue;
+          }
           if (!nsub) {
             if (best < 0 || h < best) best = h;
             continue;
@@ -288,6 +316,7 @@ int oracle_simulate(
         if (f > mkspan) mkspan = f;
         if (cls[v] >= 0) busy_acc[cls[v]] += occ[v];
         if (hocc[v] >= 0) busy_acc[RC_COUNT] += hocc[v];
+        if (nocc[v] >= 0) busy_acc[RC_COUNT + 1] += nocc[v];
         if (cls[v] >= 0) { /* take any free server of the class on this SM */
           for (int64_t q = 0; q < cap[cls[v]]; q++) {
             int64_t *s = &srv[cls[v]][sm * cap[cls[v]] + q];
@@ -297,6 +326,12 @@ int oracle_simulate(
         if (hocc[v] >= 0) {
           for (int64_t q = 0; q < cap_hbm; q++)
             if (hsrv[q] <= t) { hsrv[q] = t + hocc[v]; break; }
+        }
+        if (nocc[v] >= 0) { /* any free NoC server of the SM's group */
+          for (int64_t q = 0; q < cap_noc; q++) {
+            int64_t *s = &nsrv[(sm / csms) * cap_noc + q];
+            if (*s <= t) { *s = t + nocc[v]; break; }
+          }
         }
         for (e = row_ptr[v]; e < (int64_t)row_ptr[v + 1]; e++) {
           const int64_t u = col[e];
@@ -327,6 +362,9 @@ int oracle_simulate(
         if (srv[r][k] > t && srv[r][k] < tn) tn = srv[r][k];
     for (k = 0; k < cap_hbm; k++)
       if (hsrv[k] > t && hsrv[k] < tn) tn = hsrv[k];
+    if (noc)
+      for (k = 0; k < ngrp * cap_noc; k++)
+        if (nsrv[k] > t && nsrv[k] < tn) tn = nsrv[k];
     if (nsub)
       for (k = 0; k < nq; k++)
         if (sub_avail[k] > t && sub_avail[k] < tn) tn = sub_avail[k];
@@ -335,12 +373,12 @@ int oracle_simulate(
   }
   *makespan = mkspan;
   if (busy)
-    for (r = 0; r <= RC_COUNT; r++) busy[r] = busy_acc[r];
+    for (r = 0; r < RC_COUNT + 2; r++) busy[r] = busy_acc[r];
 
 out:
   free(cls); free(occ); free(hocc); free(lat); free(npend); free(rdy); free(nxt); free(head);
   free(rem); free(endt); free(sm_of); free(res); free(res_cnt); free(hsrv);
-  free(slot_of); free(sub_avail); free(sub_last); free(cand); free(cand_key);
+  free(slot_of); free(sub_avail); free(sub_last); free(cand); free(cand_key); free(nsrv); free(nocc);
   for (r = 0; r < RC_COUNT; r++) free(srv[r]);
   return status;
 }

@@ -57,7 +57,7 @@ class Result:
     start: np.ndarray    # int64 [n]
     finish: np.ndarray   # int64 [n]
     cta_sm: np.ndarray   # int32 [C]
-    busy: np.ndarray = None  # int64 [6]: busy server-cycles of TENSOR, TMA, LSU, ALU, BAR, HBM
+    busy: np.ndarray = None  # int64 [7]: busy server-cycles of TENSOR, TMA, LSU, ALU, BAR, HBM, NoC
 
 
 def _ptr(a):
@@ -82,7 +82,7 @@ def simulate_arrays(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_
     finish = np.empty(max(n, 1), np.int64)
     cta_sm = np.empty(max(C, 1), np.int32)
     mk = ctypes.c_int64(0)
-    busy = np.zeros(6, np.int64)
+    busy = np.zeros(7, np.int64)
     st = lib.oracle_simulate(n, m, C, int(warps_per_cta), _ptr(a["row_ptr"]), _ptr(a["col"]), _ptr(a["ekind"]),
                              _ptr(a["type"]), _ptr(a["warp"]), _ptr(a["cta"]), _ptr(a["work"]),
                              _ptr(a["lat_extra"]), _ptr(a["cta_kernel"]), _ptr(prm), _ptr(start), _ptr(finish),

@@ -18,15 +18,17 @@ Pure Python; only for graphs of a few dozen nodes with short latencies.
 """
 from __future__ import annotations
 
-LOAD, SMEM, MMA, EW, STORE, BAR, NOP = range(7)
+LOAD, SMEM, MMA, EW, STORE, BAR, NOP, DSMEM = range(8)
 ISSUE = 1
 
 
 def node_costs(ty, work, lat_extra, prm):
-    """(per-SM class or None, its occupancy, HBM occupancy or None, latency)."""
+    """(per-SM class or None, its occupancy, HBM occupancy or None, NoC
+    occupancy or None, latency)."""
     def cdiv(a, b):
         return -(-a // b)
     num = {"hbm": prm[2], "tma": prm[4], "smem": prm[6], "mma": prm[8], "alu": prm[10]}
+    nocc = None
     if ty == LOAD:
         cls, occ, hocc, base = "tma", cdiv(work, num["tma"]), cdiv(work, num["hbm"]), prm[5] + prm[3]
     elif ty == STORE:
@@ -39,10 +41,13 @@ def node_costs(ty, work, lat_extra, prm):
         cls, occ, hocc, base = "alu", cdiv(work, num["alu"]), None, prm[11]
     elif ty == BAR:
         cls, occ, hocc, base = "bar", 1, None, prm[12]
+    elif ty == DSMEM:   # the local shared-memory port plus the SM group's NoC
+        cls, occ, hocc, base = "lsu", cdiv(work, num["smem"]), None, prm[7] + prm[23]
+        nocc = cdiv(work, prm[22])
     else:
         cls, occ, hocc, base = None, 0, None, 0
-    lat = base + lat_extra + max([0] + ([occ] if cls else []) + ([hocc] if hocc is not None else []))
-    return cls, occ, hocc, lat
+    lat = base + lat_extra + max([0] + ([occ] if cls else []) + [x for x in (hocc, nocc) if x is not None])
+    return cls, occ, hocc, nocc, lat
 
 
 def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel, warps_per_cta, prm,
@@ -59,6 +64,7 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     per = cps * warps_per_cta
     cap = {"tensor": prm[13], "tma": prm[14], "lsu": prm[15], "alu": prm[16], "bar": prm[17]}
     cap_hbm = prm[18]
+    cap_noc, group = prm[24], prm[25]
     costs = [node_costs(int(type_[v]), int(work[v]), int(lat_extra[v]), prm) for v in range(n)]
     preds = [[] for _ in range(n)]
     for u in range(n):
@@ -69,12 +75,12 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     cta_sm = [-1] * C
     cta_slot = [-1] * C
     launched = [False] * C
-    total_lat = sum(c[3] for c in costs)
+    total_lat = sum(c[4] for c in costs)
     if t_limit is None:   # every cycle without an issue lies under some node's latency or issue slot
         t_limit = total_lat + n + 2
 
     def finish(v):
-        return start[v] + costs[v][3]
+        return start[v] + costs[v][4]
 
     def retired(c, t):
         return launched[c] and all(start[v] is not None and finish(v) <= t for v in members[c])
@@ -95,6 +101,10 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     def busy_hbm(t):
         return sum(1 for u in range(n) if start[u] is not None and costs[u][2] is not None
                    and start[u] <= t < start[u] + costs[u][2])
+
+    def busy_noc(grp, t):
+        return sum(1 for u in range(n) if start[u] is not None and costs[u][3] is not None
+                   and cta_sm[int(cta[u])] // group == grp and start[u] <= t < start[u] + costs[u][3])
 
     def sched(v):
         """(SM, scheduler, warp slot) of node v's warp."""
@@ -133,10 +143,12 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
             rel = max(rel, start[u] if k == ISSUE else finish(u))
         if rel > t:
             return False
-        cls, _occ, hocc, _lat = costs[v]
+        cls, _occ, hocc, nocc, _lat = costs[v]
         if cls is not None and busy(cls, cta_sm[c], t) >= cap[cls]:
             return False
         if hocc is not None and busy_hbm(t) >= cap_hbm:
+            return False
+        if nocc is not None and busy_noc(cta_sm[c] // group, t) >= cap_noc:
             return False
         return True
 
@@ -181,24 +193,27 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
             return -8, 0, start, [None] * n, cta_sm
 
 
-CLASS_ORDER = ("tensor", "tma", "lsu", "alu", "bar", "hbm")
+CLASS_ORDER = ("tensor", "tma", "lsu", "alu", "bar", "hbm", "noc")
 
 
 def busy_cycles(type_, work, lat_extra, prm, start, makespan):
     """Busy server-cycles of each class, measured on a finished schedule by
     sweeping every cycle t in [0, makespan) and counting the servers held at t
-    (a node holds one server of its class on [start, start + occupancy), and
-    one HBM server on [start, start + HBM occupancy)).  Returned in the order
-    TENSOR, TMA, LSU, ALU, BAR, HBM."""
+    (a node holds one server of its class on [start, start + occupancy), one
+    HBM server on [start, start + HBM occupancy) and one NoC server on
+    [start, start + NoC occupancy)).  Returned in the order TENSOR, TMA, LSU,
+    ALU, BAR, HBM, NoC."""
     prm = [int(x) for x in prm]
     costs = [node_costs(int(type_[v]), int(work[v]), int(lat_extra[v]), prm) for v in range(len(type_))]
     total = dict.fromkeys(CLASS_ORDER, 0)
     for t in range(makespan):
-        for v, (cls, occ, hocc, _lat) in enumerate(costs):
+        for v, (cls, occ, hocc, nocc, _lat) in enumerate(costs):
             if cls is not None and start[v] <= t < start[v] + occ:
                 total[cls] += 1
             if hocc is not None and start[v] <= t < start[v] + hocc:
                 total["hbm"] += 1
+            if nocc is not None and start[v] <= t < start[v] + nocc:
+                total["noc"] += 1
     return [total[k] for k in CLASS_ORDER]
 
 

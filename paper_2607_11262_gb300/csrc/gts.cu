@@ -74,12 +74,16 @@ constexpr uint32_t DEG_BIG = 31;            // successor count field: 31 = read 
 
 // per-SM resource classes (Section 5.2)
 enum : uint32_t { RC_TENSOR = 0, RC_TMA = 1, RC_LSU = 2, RC_ALU = 3, RC_BAR = 4, RC_N = 5, RC_NONE = 7 };
-// Per node type (LOAD, SMEM, MMA, EW, STORE, BAR, NOP), one nibble each:
-// its per-SM class, and the rate that sets its occupancy (0 HBM, 1 TMA,
-// 2 SMEM, 3 MMA, 4 ALU, 5 = one cycle, 6 = none).  LOAD and STORE also take
-// an HBM server.
-constexpr uint32_t TYPE_CLASS = 0x7413021u;
-constexpr uint32_t TYPE_RATE = 0x6514321u;
+// class code of a DSMEM node: an LSU server on its SM plus a NoC server of its SM group
+constexpr uint32_t RC_DSM = 5;
+// class_mask bit: some node crosses the NoC (servers of unused classes are not kept)
+constexpr uint32_t CM_NOC = 1u << 5;
+// Per node type (LOAD, SMEM, MMA, EW, STORE, BAR, NOP, DSMEM), one nibble
+// each: its class code, and the rate that sets its per-SM occupancy (0 HBM,
+// 1 TMA, 2 SMEM, 3 MMA, 4 ALU, 5 = one cycle, 6 = none).  LOAD and STORE also
+// take an HBM server.
+constexpr uint32_t TYPE_CLASS = 0x57413021u;
+constexpr uint32_t TYPE_RATE = 0x26514321u;
 constexpr uint32_t TYPE_HBM = 0x11u;
 static_assert(GTS_P_TMA_BPC == GTS_P_HBM_BPC + 2 && GTS_P_SMEM_BPC == GTS_P_HBM_BPC + 4 &&
                   GTS_P_MMA_FMA_PC == GTS_P_HBM_BPC + 6 && GTS_P_ALU_OPS_PC == GTS_P_HBM_BPC + 8,
@@ -120,7 +124,7 @@ struct DevGraph {
   const uint32_t *node_off;    // [G+1]
   const uint32_t *cta_off;     // [G+1]
   uint32_t W, G, row_nodes, row_ctas, cross_cta;
-  uint32_t class_mask;  // bit r: some node uses per-SM class r (servers of unused classes are not kept)
+  uint32_t class_mask;  // bit r < 5: some node uses per-SM class r; CM_NOC: some node crosses the NoC
 };
 
 // ----------------------------------------------------------------- per-point layout
@@ -128,9 +132,9 @@ struct DevGraph {
 // warp; CTA slot j lives on SM j / ctas_per_sm (SM-major, so the lowest free
 // slot is on the lowest SM with room).  Only min(num_sms*cps, C) CTA slots can
 // ever be occupied (a launch always takes the lowest free slot).
-constexpr uint32_t O_MAG = GTS_NPARAM;       // 5 x 2 words: division constants of the rates (8-byte aligned)
-constexpr uint32_t O_BASE = GTS_NPARAM + 10; // 8 words: base latency per node type
-constexpr uint32_t O_DYN = GTS_NPARAM + 18;  // first per-point array
+constexpr uint32_t O_MAG = GTS_NPARAM;       // 6 x 2 words: division constants of the 5 rates and the NoC rate
+constexpr uint32_t O_BASE = GTS_NPARAM + 12; // 8 words: base latency per node type
+constexpr uint32_t O_DYN = GTS_NPARAM + 20;  // first per-point array
 static_assert(O_MAG % 2 == 0, "division constants are 8-byte words");
 // slot record (5 words): id|HBM, rdy, pending<<8 | deg<<3 | class, next, successor begin
 constexpr uint32_t F_HID = 0, F_RDY = 1, F_META = 2, F_NXT = 3, F_SB = 4, SLOT_WORDS = 5;
@@ -145,11 +149,11 @@ constexpr uint32_t C_ID = 0, C_REM = 1, C_END = 2, CTA_WORDS = 3;
 constexpr uint32_t Q_AVAIL = 0, Q_LAST = 1, SUB_WORDS = 2;
 
 struct Layout {
-  uint32_t S, Scta, NS, SC, cap_hbm, per, nsub;
-  uint32_t o_slot, o_sm, o_cta, o_sv, o_hs, o_sub, words;
+  uint32_t S, Scta, NS, SC, cap_hbm, per, nsub, csms, cap_noc;
+  uint32_t o_slot, o_sm, o_cta, o_sv, o_hs, o_sub, o_ns, words;
 };
 
-__host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
+__host__ __device__ inline int check_row(const int32_t *p, uint32_t G, uint32_t class_mask) {
   if (p[GTS_P_NUM_SMS] < 1 || p[GTS_P_CTAS_PER_SM] < 1) return GTS_ERR_INVALID_PARAMS;
   for (int i = 0; i < 5; i++)
     if (p[GTS_P_HBM_BPC + 2 * i] < 1) return GTS_ERR_INVALID_PARAMS;
@@ -167,7 +171,15 @@ __host__ __device__ inline int check_row(const int32_t *p, uint32_t G) {
   } else {
     return GTS_ERR_INVALID_PARAMS;
   }
-  for (int i = GTS_P_SUBPARTITIONS + 1; i < GTS_NPARAM; i++)
+  const int32_t csms = p[GTS_P_CLUSTER_SMS], cap_noc = p[GTS_P_CAP_NOC];
+  if (csms != 0) {
+    if (p[GTS_P_NOC_BPC] < 1 || p[GTS_P_NOC_LAT] < 0 || cap_noc < 1 || cap_noc > 32 || csms > 32)
+      return GTS_ERR_INVALID_PARAMS;
+  } else if (p[GTS_P_NOC_BPC] != 0 || p[GTS_P_NOC_LAT] != 0 || cap_noc != 0) {
+    return GTS_ERR_INVALID_PARAMS;
+  }
+  if ((class_mask & CM_NOC) && csms == 0) return GTS_ERR_INVALID_PARAMS;  // DSMEM nodes, no NoC
+  for (int i = GTS_P_CLUSTER_SMS + 1; i < GTS_NPARAM; i++)
     if (p[i] != 0) return GTS_ERR_INVALID_PARAMS;
   return GTS_OK;
 }
@@ -204,6 +216,10 @@ __host__ __device__ inline bool make_layout(const int32_t *p, uint32_t CG, uint3
   L.o_hs = (uint32_t)w; w += L.cap_hbm;
   L.nsub = (uint32_t)p[GTS_P_SUBPARTITIONS];
   L.o_sub = (uint32_t)w; w += (uint64_t)L.NS * L.nsub * SUB_WORDS;
+  L.csms = (uint32_t)p[GTS_P_CLUSTER_SMS];
+  L.cap_noc = (class_mask & CM_NOC) ? (uint32_t)p[GTS_P_CAP_NOC] : 0u;
+  L.o_ns = (uint32_t)w;  // NoC servers per SM group
+  if (L.cap_noc) w += (uint64_t)((L.NS + L.csms - 1) / L.csms) * L.cap_noc;
   w = (w + 3) & ~(uint64_t)3;  // 16-byte multiple
   if (w * 4 > MAX_SMEM_BYTES) return false;
   L.words = (uint32_t)w;
@@ -263,18 +279,23 @@ struct Pt {
   }
 };
 
-// Occupancies and latency of a node (Section 5.2 throughput model).
+// Occupancies and latency of a node (Section 5.2 throughput model): per-SM
+// class, HBM and NoC occupancy; latency = base + lat_extra + the largest.
+template <bool EXT>
 __device__ __forceinline__ void node_cost(const uint32_t *sp, uint32_t type, uint32_t work, uint32_t lx,
-                                          uint32_t &occ, uint32_t &hocc, uint64_t &lat) {
+                                          uint32_t &occ, uint32_t &hocc, uint32_t &nocc, uint64_t &lat) {
   const uint32_t rt = (TYPE_RATE >> (4 * type)) & 15u;
   occ = rt == 5u ? 1u : 0u;
   if (rt < 5u) occ = cdiv_c(work, sp[GTS_P_HBM_BPC + 2 * rt], *reinterpret_cast<const uint64_t *>(sp + O_MAG + 2 * rt));
   hocc = 0u;
   if ((TYPE_HBM >> type) & 1u) hocc = cdiv_c(work, sp[GTS_P_HBM_BPC], *reinterpret_cast<const uint64_t *>(sp + O_MAG));
-  lat = (uint64_t)sp[O_BASE + type] + lx + (occ > hocc ? occ : hocc);
+  nocc = 0u;
+  if (EXT && type == GTS_DSMEM) nocc = cdiv_c(work, sp[GTS_P_NOC_BPC], *reinterpret_cast<const uint64_t *>(sp + O_MAG + 10));
+  lat = (uint64_t)sp[O_BASE + type] + lx + max(max(occ, hocc), nocc);
 }
 
 // Key of slot i computed at cycle t (>= t; INF if it cannot issue yet).
+template <bool EXT>
 __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t) {
   const uint32_t *sl = P.slot(i);
   const uint32_t h = sl[F_HID];
@@ -284,11 +305,18 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
   const uint32_t cls = meta & 7u;
   if (cls != RC_NONE) {
     const uint32_t sm = i / P.L.per;
-    const uint32_t *sv = P.sp + P.L.o_sv + sm * P.L.SC + P.cls_off(cls);
-    const uint32_t cap = P.cls_cap(cls);
+    const uint32_t sc = EXT && cls == RC_DSM ? RC_LSU : cls;
+    const uint32_t *sv = P.sp + P.L.o_sv + sm * P.L.SC + P.cls_off(sc);
+    const uint32_t cap = P.cls_cap(sc);
     uint32_t a = sv[0];
     for (uint32_t q = 1; q < cap; q++) a = min(a, sv[q]);
     k = max(k, a);
+    if (EXT && cls == RC_DSM) {  // and a NoC server of the SM's group
+      const uint32_t *ns = P.sp + P.L.o_ns + (sm / P.L.csms) * P.L.cap_noc;
+      a = ns[0];
+      for (uint32_t q = 1; q < P.L.cap_noc; q++) a = min(a, ns[q]);
+      k = max(k, a);
+    }
   }
   return k;
 }
@@ -298,6 +326,7 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
 // E_u = max(first cycle it may issue, least effective key of its heads); its
 // pick is the first head in policy order among those whose effective key is
 // <= E_u.  The record holds the least (E_u, id of the pick) over u.
+template <bool EXT>
 __device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
   const uint32_t per = P.L.per, nsub = P.L.nsub, i0 = s * per;
   const uint32_t nl = min(per, P.L.S - i0);
@@ -307,7 +336,7 @@ __device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t 
     const uint32_t *sq = P.sub(s, u);
     uint32_t m = INF;
     for (uint32_t l = u; l < nl; l += nsub) {
-      const uint32_t k = slot_key(P, i0 + l, t);
+      const uint32_t k = slot_key<EXT>(P, i0 + l, t);
       if (k == INF) continue;
       if (P.slot(i0 + l)[F_HID] & HBM_BIT) {
         hmin = min(hmin, k);
@@ -320,7 +349,7 @@ __device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t 
     const uint32_t E = max(m, sq[Q_AVAIL]), last = sq[Q_LAST];
     uint64_t bp = INF64;  // (policy key << 32 | slot)
     for (uint32_t l = u; l < nl; l += nsub) {
-      const uint32_t k = slot_key(P, i0 + l, t);
+      const uint32_t k = slot_key<EXT>(P, i0 + l, t);
       if (k == INF) continue;
       const uint32_t e = (P.slot(i0 + l)[F_HID] & HBM_BIT) ? max(k, H) : k;
       if (e > E) continue;
@@ -348,10 +377,10 @@ __device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t 
 
 // Warp-parallel: the keys of SM s's heads at cycle t and the SM's summary
 // record.  All lanes call it.
-template <bool SCHED>
+template <bool EXT>
 __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane) {
-  if (SCHED && P.L.nsub) {
-    if (lane == 0) rescan_sm_sub(P, s, t, H);
+  if (EXT && P.L.nsub) {
+    if (lane == 0) rescan_sm_sub<EXT>(P, s, t, H);
     __syncwarp();
     return;
   }
@@ -362,7 +391,7 @@ __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, 
     const uint32_t i = base + lane;
     uint64_t val = INF64;
     if (i < i1) {
-      const uint32_t k = slot_key(P, i, t);
+      const uint32_t k = slot_key<EXT>(P, i, t);
       const uint32_t h = P.slot(i)[F_HID];
       if (k != INF) {
         const bool hb = (h & HBM_BIT) != 0u;
@@ -389,17 +418,17 @@ __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, 
 }
 
 // One lane: recompute the record of SM s at cycle t and horizon H.
-template <bool SCHED>
+template <bool EXT>
 __device__ __forceinline__ void rescan_sm_lane(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
-  if (SCHED && P.L.nsub) {
-    rescan_sm_sub(P, s, t, H);
+  if (EXT && P.L.nsub) {
+    rescan_sm_sub<EXT>(P, s, t, H);
     return;
   }
   const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
   uint64_t best = INF64;
   uint32_t bsl = 0, hmin = INF;
   for (uint32_t i = i0; i < i1; i++) {
-    const uint32_t k = slot_key(P, i, t);
+    const uint32_t k = slot_key<EXT>(P, i, t);
     if (k == INF) continue;
     const uint32_t h = P.slot(i)[F_HID];
     const bool hb = (h & HBM_BIT) != 0u;
@@ -477,7 +506,7 @@ struct Clock {
 
 // Retire finished CTAs and launch as many CTAs as fit at cycle t (Section 5.1
 // TB scheduler; kernel-boundary gate).  Returns false on step-limit.
-template <bool SCHED>
+template <bool EXT>
 __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_row, int lane, uint64_t &b,
                             uint32_t &bsl) {
   const uint32_t t = C.t;
@@ -534,15 +563,16 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
     }
     __syncwarp();
     const uint32_t s = freeslot / P.cps;
-    refresh_sm<SCHED>(P, s, t, C.H, lane);
+    refresh_sm<EXT>(P, s, t, C.H, lane);
     refresh_owner(P, s & 31u, lane, b, bsl);
     C.next_cta++;
   }
 }
 
-// SCHED: the kernel instance that also runs the per-subpartition issue
-// policies; the host launches the plain instance when no row asks for them.
-template <bool SCHED>
+// EXT: the kernel instance that also runs the per-subpartition issue policies
+// and the NoC of DSMEM nodes; the host launches the plain instance when no row
+// asks for a policy and the graph has no DSMEM node.
+template <bool EXT>
 __global__ void __launch_bounds__(MAX_WPB * 32, 1)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
@@ -564,7 +594,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     if (lane < GTS_NPARAM) sp[lane] = (uint32_t)params[(size_t)p * GTS_NPARAM + lane];
     __syncwarp();
     const int32_t *prm = reinterpret_cast<const int32_t *>(sp);
-    int status = check_row(prm, g.G);
+    int status = check_row(prm, g.G, g.class_mask);
     const uint32_t gi = status == GTS_OK ? (uint32_t)prm[GTS_P_GRAPH_INDEX] : 0u;
     P.n0 = g.node_off[gi];
     const uint32_t nG = g.node_off[gi + 1] - P.n0;
@@ -572,7 +602,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     P.c1 = g.cta_off[gi + 1];
     const uint32_t CG = P.c1 - P.c0;
     if (status == GTS_OK) {
-      if (!make_layout(prm, CG, P.W, g.class_mask, P.L) || P.L.words > budget_words || (!SCHED && P.L.nsub))
+      if (!make_layout(prm, CG, P.W, g.class_mask, P.L) || P.L.words > budget_words ||
+          (!EXT && (P.L.nsub || P.L.cap_noc)))
         status = GTS_ERR_UNSUPPORTED;
     }
     if (status != GTS_OK) {
@@ -606,6 +637,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     }
     if (lane < (int)RC_N) {
       *reinterpret_cast<uint64_t *>(sp + O_MAG + 2 * lane) = div_const((uint32_t)prm[GTS_P_HBM_BPC + 2 * lane]);
+    } else if (lane == (int)RC_N) {
+      *reinterpret_cast<uint64_t *>(sp + O_MAG + 10) = div_const((uint32_t)prm[GTS_P_NOC_BPC]);
     }
     if (lane < 8) {  // base latency per type: LOAD, SMEM, MMA, EW, STORE, BAR, NOP
       uint32_t bl = 0;
@@ -616,6 +649,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         case GTS_EW: bl = (uint32_t)prm[GTS_P_ALU_LAT]; break;
         case GTS_STORE: bl = (uint32_t)prm[GTS_P_TMA_LAT]; break;
         case GTS_BAR: bl = (uint32_t)prm[GTS_P_BAR_LAT]; break;
+        case GTS_DSMEM: bl = (uint32_t)prm[GTS_P_SMEM_LAT] + (uint32_t)prm[GTS_P_NOC_LAT]; break;
         default: break;
       }
       sp[O_BASE + lane] = bl;
@@ -632,6 +666,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     for (uint32_t j = lane; j < P.L.Scta; j += 32) P.cta(j)[C_ID] = NONE;
     for (uint32_t k = lane; k < P.L.NS * P.L.SC; k += 32) sp[P.L.o_sv + k] = 0u;
     for (uint32_t k = lane; k < P.L.cap_hbm; k += 32) sp[P.L.o_hs + k] = 0u;
+    if (P.L.cap_noc)
+      for (uint32_t k = lane; k < ((P.L.NS + P.L.csms - 1) / P.L.csms) * P.L.cap_noc; k += 32) sp[P.L.o_ns + k] = 0u;
     for (uint32_t k = lane; k < P.L.NS * P.L.nsub; k += 32) {
       sp[P.L.o_sub + k * SUB_WORDS + Q_AVAIL] = 0u;
       sp[P.L.o_sub + k * SUB_WORDS + Q_LAST] = NONE;
@@ -660,7 +696,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     uint64_t busy = 0;  // lane r < 5: server-cycles of per-SM class r; lane 5: HBM
     uint64_t b = INF64;  // this lane's best (effective cycle << 32 | id) over its SMs
     uint32_t bsl = 0;    // ... and its slot
-    if (!launch_ctas<SCHED>(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
+    if (!launch_ctas<EXT>(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
 
     while (status == GTS_OK && issued < nG) {
       // ---- next event: minimum of (effective cycle, node id) over all heads
@@ -673,7 +709,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
         C.t = tn;
         if (C.next_ret <= C.t) {  // a CTA retires first: launch, then choose again
-          if (!launch_ctas<SCHED>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
+          if (!launch_ctas<EXT>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
           continue;
         }
         // otherwise the minimum just found is the first issue at the new cycle
@@ -702,23 +738,33 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       if (deg == DEG_BIG) deg = g.rng[v].w - sb;
       uint2 ew = make_uint2(NONE, 0);
       if ((uint32_t)lane < deg) ew = g.succ[sb + lane];
-      uint32_t occ, hocc;
+      uint32_t occ, hocc, nocc;
       uint64_t lat;
-      node_cost(sp, rv.w & 15u, rv.x, rv.y, occ, hocc, lat);
+      node_cost<EXT>(sp, rv.w & 15u, rv.x, rv.y, occ, hocc, nocc, lat);
       const uint64_t f64 = (uint64_t)t + lat;
       if (f64 > 0x7FFFFFFFull) { status = GTS_ERR_OVERFLOW; break; }
       const uint32_t f = (uint32_t)f64;
-      busy += (uint32_t)lane == cls ? occ : ((uint32_t)lane == RC_N ? hocc : 0u);
+      const uint32_t scls = EXT && cls == RC_DSM ? RC_LSU : cls;  // the per-SM class it takes
+      busy += (uint32_t)lane == scls ? occ
+            : (uint32_t)lane == GTS_BUSY_HBM ? hocc : ((uint32_t)lane == GTS_BUSY_NOC ? nocc : 0u);
       cn.x = __shfl_sync(FULL, cn.x, 0);
       cn.y = __shfl_sync(FULL, cn.y, 0);
       // take one free server of the node's class on its SM (lane k tests server k)
       if (cls != RC_NONE) {
-        uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + P.cls_off(cls);
-        const bool fr = (uint32_t)lane < P.cls_cap(cls) && sv[lane] <= t;
+        uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + P.cls_off(scls);
+        const bool fr = (uint32_t)lane < P.cls_cap(scls) && sv[lane] <= t;
         const uint32_t bal = __ballot_sync(FULL, fr);
         if (lane == __ffs(bal) - 1) sv[lane] = t + occ;
       }
-      if (SCHED && P.L.nsub && lane == 0) {  // the issuing scheduler: one issue per cycle, remember the slot
+      bool noc_touch = false;  // a NoC server of the SM's group was taken
+      if (EXT && cls == RC_DSM) {
+        uint32_t *ns = sp + P.L.o_ns + (sm / P.L.csms) * P.L.cap_noc;
+        const bool fr = (uint32_t)lane < P.L.cap_noc && ns[lane] <= t;
+        const uint32_t bal = __ballot_sync(FULL, fr);
+        if (lane == __ffs(bal) - 1) ns[lane] = t + nocc;
+        noc_touch = P.L.csms > 1u;
+      }
+      if (EXT && P.L.nsub && lane == 0) {  // the issuing scheduler: one issue per cycle, remember the slot
         const uint32_t l = i - sm * P.L.per;
         uint32_t *sq = P.sub(sm, l % P.L.nsub);
         sq[Q_AVAIL] = t + 1u;
@@ -803,17 +849,17 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
       if (cross_touch) {  // a release reached a head of another CTA: recompute everything
-        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane<SCHED>(P, s, t, C.H);
+        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane<EXT>(P, s, t, C.H);
         __syncwarp();
         b = lane_best(P, lane, bsl);
       } else {
-        refresh_sm<SCHED>(P, sm, t, C.H, lane);
+        refresh_sm<EXT>(P, sm, t, C.H, lane);
         if (C.H != prevH) {
           // SMs whose HBM heads H overtakes change their effective cycles
           bool any = false;
           for (uint32_t s = lane; s < P.L.NS; s += 32) {
             if (s != sm && P.smrec(s)[3] < C.H) {
-              rescan_sm_lane<SCHED>(P, s, t, C.H);
+              rescan_sm_lane<EXT>(P, s, t, C.H);
               any = true;
             }
           }
@@ -821,11 +867,20 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         } else {
           refresh_owner(P, sm & 31u, lane, b, bsl);
         }
+        if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
+          const uint32_t g0 = (sm / P.L.csms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
+          for (uint32_t s = g0 + lane; s < g1; s += 32)
+            if (s != sm) rescan_sm_lane<EXT>(P, s, t, C.H);
+          __syncwarp();
+          bool mine = false;  // this lane owns one of them
+          for (uint32_t s = g0; s < g1; s++) mine |= s != sm && (s & 31u) == (uint32_t)lane;
+          if (mine) b = lane_best(P, lane, bsl);
+        }
       }
       __syncwarp();
       if (rem == 0u) {
         if (cend <= t) {
-          if (!launch_ctas<SCHED>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
+          if (!launch_ctas<EXT>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
         } else {
           C.next_ret = min(C.next_ret, cend);
         }
@@ -962,9 +1017,10 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
     row_ctas = std::max(row_ctas, c1 - c0);
     for (uint32_t v = n0; v < n1; v++) {
       if (row_ptr[v + 1] < row_ptr[v]) return fail(GTS_ERR_INVALID_GRAPH, "row_ptr decreases at node " + std::to_string(v));
-      if (ty[v] > GTS_NOP) return fail(GTS_ERR_INVALID_GRAPH, "bad type at node " + std::to_string(v));
+      if (ty[v] > GTS_DSMEM) return fail(GTS_ERR_INVALID_GRAPH, "bad type at node " + std::to_string(v));
       const uint32_t cls_v = (TYPE_CLASS >> (4 * ty[v])) & 15u;
       if (cls_v < RC_N) class_mask |= 1u << cls_v;
+      if (cls_v == RC_DSM) class_mask |= (1u << RC_LSU) | CM_NOC;
       if (wp[v] >= W) return fail(GTS_ERR_INVALID_GRAPH, "warp >= warps_per_cta at node " + std::to_string(v));
       if (cta[v] < c0 || cta[v] >= c1) return fail(GTS_ERR_INVALID_GRAPH, "cta outside its graph at node " + std::to_string(v));
       for (uint32_t x = row_ptr[v]; x < row_ptr[v + 1]; x++) {
@@ -1063,7 +1119,7 @@ gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_p
   P->sched.assign(n_points, 0u);
   for (uint32_t p = 0; p < n_points; p++) {
     const int32_t *row = h.data() + (size_t)p * GTS_NPARAM;
-    if (check_row(row, g->G) != GTS_OK) continue;
+    if (check_row(row, g->G, g->dg.class_mask) != GTS_OK) continue;
     P->sched[p] = row[GTS_P_ISSUE_POLICY] != GTS_POLICY_LOWEST_ID;
     const uint32_t gi = (uint32_t)row[GTS_P_GRAPH_INDEX];
     Layout L;
@@ -1085,7 +1141,7 @@ uint64_t scratch_row_bytes(const gts_graph *g) { return (((uint64_t)g->dg.row_no
 
 struct Plan {
   uint32_t words, wpb, smem, blocks, warps;
-  bool sched;  // launch the instance with the per-subpartition policies
+  bool sched;  // launch the extended instance (issue policies, NoC)
 };
 
 gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, uint32_t np, uint32_t flags,
@@ -1097,6 +1153,7 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
     words = std::max(words, P->words[p]);
     pl.sched = pl.sched || P->sched[p];
   }
+  pl.sched = pl.sched || (g->dg.class_mask & CM_NOC) != 0u;
   const uint32_t bytes = words * 4;
   pl.words = words;
   const void *kern = pl.sched ? (const void *)k_simulate<true> : (const void *)k_simulate<false>;

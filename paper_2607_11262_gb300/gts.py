@@ -34,9 +34,9 @@ GTS_WANT_DIGEST = 2
 GTS_WANT_CTA_SM = 4
 GTS_WANT_BUSY = 8
 
-GTS_BUSY_CLASSES = 6
-GTS_BUSY_TENSOR, GTS_BUSY_TMA, GTS_BUSY_LSU, GTS_BUSY_ALU, GTS_BUSY_BAR, GTS_BUSY_HBM = range(6)
-BUSY_NAMES = ("tensor", "tma", "lsu", "alu", "bar", "hbm")
+GTS_BUSY_CLASSES = 7
+GTS_BUSY_TENSOR, GTS_BUSY_TMA, GTS_BUSY_LSU, GTS_BUSY_ALU, GTS_BUSY_BAR, GTS_BUSY_HBM, GTS_BUSY_NOC = range(7)
+BUSY_NAMES = ("tensor", "tma", "lsu", "alu", "bar", "hbm", "noc")
 
 GTS_NPARAM = 32
 GTS_POLICY_LOWEST_ID, GTS_POLICY_GTO, GTS_POLICY_RR = 0, 1, 2
@@ -339,7 +339,8 @@ def simulate(dgraph: DeviceGraph, dparams: DeviceParams, first_point=0, n_points
 def utilisation(busy, makespan, params):
     """Per-class utilisation of each point from its busy server-cycles:
     busy_r / (servers_r * makespan), servers_r = cap_r * num_sms for the per-SM
-    classes and cap_hbm for HBM; 0 where the makespan is 0.  numpy in, numpy out
+    classes, cap_hbm for HBM and cap_noc * ceil(num_sms / cluster_sms) for the
+    NoC; 0 where the makespan is 0 or the row has no NoC.  numpy in, numpy out
     ([n_points][GTS_BUSY_CLASSES] float64)."""
     import numpy as np
     busy = np.asarray(busy, np.float64)
@@ -348,5 +349,7 @@ def utilisation(busy, makespan, params):
     servers = np.empty((prm.shape[0], GTS_BUSY_CLASSES), np.float64)
     servers[:, :5] = prm[:, 13:18] * prm[:, 0:1]
     servers[:, 5] = prm[:, 18]
+    groups = np.where(prm[:, 25] > 0, -(-prm[:, 0] // np.maximum(prm[:, 25], 1)), 0)
+    servers[:, 6] = prm[:, 24] * groups
     den = servers * mk[:, None]
     return np.divide(busy, den, out=np.zeros_like(busy), where=den > 0)

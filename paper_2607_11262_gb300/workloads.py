@@ -3,7 +3,8 @@
 A tile graph (Section 4.1) is a DAG G = (V, E) whose nodes are warp-level tile
 operations and whose edges are dependencies.  Each node records
 
-* ``type``      -- its operation descriptor (LOAD, SMEM, MMA, EW, STORE, BAR, NOP),
+* ``type``      -- its operation descriptor (LOAD, SMEM, MMA, EW, STORE, BAR, NOP,
+                   DSMEM = a remote shared-memory access over the on-chip NoC),
                    which fixes the hardware unit that serves it (Section 4.1, 5.2);
 * ``warp``      -- the CTA-local logical warp (execution group) that issues it;
                    a warpgroup is one logical warp (Section 4.1);
@@ -33,20 +34,22 @@ import hashlib
 import numpy as np
 
 # ---------------------------------------------------------------- vocabulary
-LOAD, SMEM, MMA, EW, STORE, BAR, NOP = range(7)
-TYPE_NAMES = ("LOAD", "SMEM", "MMA", "EW", "STORE", "BAR", "NOP")
+LOAD, SMEM, MMA, EW, STORE, BAR, NOP, DSMEM = range(8)
+TYPE_NAMES = ("LOAD", "SMEM", "MMA", "EW", "STORE", "BAR", "NOP", "DSMEM")
 DATA, ISSUE = 0, 1
 
 NPARAM = 32
 (P_NUM_SMS, P_CTAS_PER_SM, P_HBM_BPC, P_DRAM_LAT, P_TMA_BPC, P_TMA_LAT,
  P_SMEM_BPC, P_SMEM_LAT, P_MMA_FMA_PC, P_MMA_LAT, P_ALU_OPS_PC, P_ALU_LAT,
  P_BAR_LAT, P_CAP_TENSOR, P_CAP_TMA, P_CAP_LSU, P_CAP_ALU, P_CAP_BAR,
- P_CAP_HBM, P_GRAPH_INDEX, P_ISSUE_POLICY, P_SUBPARTITIONS) = range(22)
+ P_CAP_HBM, P_GRAPH_INDEX, P_ISSUE_POLICY, P_SUBPARTITIONS, P_NOC_BPC, P_NOC_LAT, P_CAP_NOC,
+ P_CLUSTER_SMS) = range(26)
 PARAM_NAMES = ("num_sms", "ctas_per_sm", "hbm_bpc", "dram_lat", "tma_bpc",
                "tma_lat", "smem_bpc", "smem_lat", "mma_fma_pc", "mma_lat",
                "alu_ops_pc", "alu_lat", "bar_lat", "cap_tensor", "cap_tma",
                "cap_lsu", "cap_alu", "cap_bar", "cap_hbm", "graph_index",
-               "issue_policy", "subpartitions") + tuple(f"reserved{i}" for i in range(22, NPARAM))
+               "issue_policy", "subpartitions", "noc_bpc", "noc_lat", "cap_noc",
+               "cluster_sms") + tuple(f"reserved{i}" for i in range(26, NPARAM))
 # issue policies (Section 5.3): one global lowest-id order, or per-subpartition
 # greedy-then-oldest / round-robin schedulers issuing one node per cycle
 POLICY_LOWEST_ID, POLICY_GTO, POLICY_RR = 0, 1, 2
@@ -57,6 +60,20 @@ H100_CORE_HZ = 1.98e9  # H100 SXM core clock, Table "GPU configurations"
 def bytes_per_cycle(tb_per_s: float) -> int:
     """DRAM bandwidth in bytes per core cycle at the H100 core clock."""
     return int(tb_per_s * 1e12 // H100_CORE_HZ)
+
+
+def with_noc(p, noc_bpc=32, noc_lat=180, cap_noc=None, cluster_sms=16):
+    """Rows ``p`` with an on-chip NoC: SM groups of ``cluster_sms``, each with
+    ``cap_noc`` servers (default: one port per SM of the group) of ``noc_bpc``
+    bytes per cycle and ``noc_lat`` cycles.  The paper gives no NoC figures;
+    32 B/cycle and 180 cycles per DSMEM access are this framework's Hopper-like
+    choice."""
+    p = np.array(p, np.int32, copy=True)
+    p[..., P_NOC_BPC] = noc_bpc
+    p[..., P_NOC_LAT] = noc_lat
+    p[..., P_CAP_NOC] = cluster_sms if cap_noc is None else cap_noc
+    p[..., P_CLUSTER_SMS] = cluster_sms
+    return p
 
 
 def default_params() -> np.ndarray:

@@ -11,6 +11,8 @@
   optimum of P|prec|Cmax;
 * per-subpartition issue policies (greedy-then-oldest, round-robin): hand
   schedules, stepper == oracle, one issue per scheduler per cycle;
+* DSMEM nodes over the on-chip NoC of SM groups: hand schedules, stepper ==
+  oracle, parameter checks;
 * busy server-cycles: equal to the stepper's cycle-by-cycle count of held
   servers; a single saturated server is busy for the whole makespan; busy
   cycles never exceed servers x makespan;
@@ -95,6 +97,54 @@ def test_golden_issue_policies():
         assert r.status == 0, case["name"]
         assert list(r.start) == case["start"], (case["name"], list(r.start))
         assert_same(r, s)
+
+
+def test_golden_noc():
+    spec = json.load(open(os.path.join(GOLDEN, "noc.json")))
+    for case in spec["cases"]:
+        nodes = case["nodes"]
+        g = TG.make(len(nodes), [], [TYPE[x[0]] for x in nodes], [x[1] for x in nodes], [x[2] for x in nodes],
+                    case["warps_per_cta"], work=[x[3] for x in nodes])
+        prm = W.with_noc(TG.unit_params(case["num_sms"], case["ctas_per_sm"]), *case["noc"])
+        if "smem_bpc" in case:
+            prm[W.P_SMEM_BPC] = case["smem_bpc"]
+        r, s = both(g, prm)
+        assert r.status == 0, case["name"]
+        assert list(r.start) == case["start"], (case["name"], list(r.start))
+        assert list(r.finish) == case["finish"], case["name"]
+        assert r.makespan == case["makespan"], case["name"]
+        assert r.busy[6] == sum(-(-x[3] // case["noc"][0]) for x in nodes if x[0] == "DSMEM")
+        assert_same(r, s)
+
+
+def test_stepper_equals_oracle_noc():
+    rng = np.random.default_rng(60)
+    types = (W.LOAD, W.SMEM, W.MMA, W.EW, W.BAR, W.NOP, W.DSMEM, W.DSMEM)
+    for i in range(140):
+        n = int(rng.integers(2, 20))
+        g = TG.random_graph(rng, n, p_edge=float(rng.uniform(0.05, 0.3)), cta_major=bool(i % 3),
+                            kernels=bool(i % 4 == 0), types=types)
+        prm = TG.small_params(rng)
+        prm = W.with_noc(prm, int(rng.integers(1, 4)), int(rng.integers(0, 4)), int(rng.integers(1, 3)),
+                         int(rng.integers(1, 4)))
+        if i % 3 == 1:
+            prm = _with_policy(prm, int(rng.integers(1, 3)), int(rng.integers(1, 4)))
+        r, s = both(g, prm)
+        assert_same(r, s)
+
+
+def test_noc_parameter_checks():
+    g = TG.make(2, [], [W.DSMEM, W.NOP], [0, 0], [0, 0], 1, work=[4, 0])
+    h = TG.make(2, [], [W.SMEM, W.NOP], [0, 0], [0, 0], 1, work=[4, 0])
+    base = TG.unit_params(1, 1)
+    assert run.simulate(g, base).status == run.ERR_INVALID_PARAMS        # DSMEM node, no NoC
+    assert run.simulate(h, base).status == 0                              # no DSMEM node, no NoC
+    assert run.simulate(g, W.with_noc(base, 1, 0, 1, 1)).status == 0
+    for fields in ((0, 0, 1, 1), (1, -1, 1, 1), (1, 0, 0, 1), (1, 0, 33, 1), (1, 0, 1, 33), (1, 0, 1, 0),
+                   (0, 5, 0, 0)):
+        prm = base.copy()
+        prm[W.P_NOC_BPC:W.P_CLUSTER_SMS + 1] = fields
+        assert run.simulate(h, prm).status == run.ERR_INVALID_PARAMS, fields
 
 
 def _with_policy(prm, policy, nsub):
@@ -282,7 +332,7 @@ def test_single_server_no_idle():
         assert r.status == 0
         assert r.makespan == int(g.work.sum())
         assert r.busy[0] == r.makespan          # the tensor server never idles
-        assert list(r.busy[1:]) == [0] * 5
+        assert list(r.busy[1:]) == [0] * 6
 
 
 # ------------------------------------------------------------------ bounds and invariants
