@@ -1,5 +1,6 @@
-"""Software-pipelining case study and tile-graph ablation on the GPU
-(Section 7.1 "Software Pipelining Impact"; Section 6.4 ablation).
+"""Case studies on the GPU: software pipelining and the tile-graph ablation
+(Section 7.1 "Software Pipelining Impact"; Section 6.4 ablation), and
+NoC-enabled fusion (Section 7.2).
 
 Every (organisation, tile, ablation) graph of ``pipelines.study_set`` runs on
 one simulated Hopper SM through libgts; the table reports, per graph, the
@@ -9,7 +10,11 @@ organisation of the same tile.  With ``--points-per-graph`` > 1 the extra
 design points sweep DRAM bandwidth and tensor rate, and the table adds the
 utilisation's minimum, mean and maximum over the sweep.
 
-    python -m paper_2607_11262_gb300.study [--points-per-graph 64] [--json out.json]
+The NoC study runs the cluster-fused attention decode of ``clusters`` with
+NoC and with DRAM exchanges for every cluster size and reports both makespans,
+the speedup and the NoC utilisation (busy NoC cycles / (servers x makespan)).
+
+    python -m paper_2607_11262_gb300.study [--study pipelines|noc] [--points-per-graph 64] [--json out.json]
 """
 from __future__ import annotations
 
@@ -18,7 +23,7 @@ import json
 
 import numpy as np
 
-from . import gts, pipelines
+from . import clusters, gts, pipelines
 
 
 def run_study(points_per_graph=1, device="cuda"):
@@ -57,6 +62,47 @@ def run_study(points_per_graph=1, device="cuda"):
     return rows
 
 
+def run_noc_study(points_per_graph=1, device="cuda"):
+    """NoC-vs-DRAM fusion study; one dict per cluster size, makespans of the
+    default point and the speedup over the sweep (min / mean / max)."""
+    import torch
+    gts.load()
+    graph, cases = clusters.study_set()
+    params = clusters.study_params(cases, points_per_graph=points_per_graph)
+    dg = gts.DeviceGraph(graph, device=device)
+    dp = gts.DeviceParams(dg, params)
+    out = gts.simulate(dg, dp, flags=gts.GTS_WANT_BUSY)
+    torch.cuda.synchronize()
+    status = out.status.cpu().numpy()
+    if np.any(status != gts.GTS_OK):
+        raise gts.GtsError(int(status[status != 0][0]), "a study point did not simulate")
+    mk = out.makespan.cpu().numpy().reshape(len(cases), points_per_graph)
+    util = gts.utilisation(out.busy.cpu().numpy(), out.makespan.cpu().numpy(), params)
+    util = util.reshape(len(cases), points_per_graph, gts.GTS_BUSY_CLASSES)
+    dp.close()
+    dg.close()
+    rows = []
+    for k in clusters.CLUSTER_SIZES:
+        a, b = cases.index((k, "noc")), cases.index((k, "dram"))
+        sp = mk[b] / mk[a]
+        rows.append(dict(cluster=k, noc_makespan=int(mk[a][0]), dram_makespan=int(mk[b][0]),
+                         speedup=float(sp[0]), speedup_min=float(sp.min()), speedup_mean=float(sp.mean()),
+                         speedup_max=float(sp.max()), noc_util=float(util[a][0, gts.GTS_BUSY_NOC]),
+                         hbm_util_noc=float(util[a][0, gts.GTS_BUSY_HBM]),
+                         hbm_util_dram=float(util[b][0, gts.GTS_BUSY_HBM])))
+    return rows
+
+
+def format_noc_table(rows):
+    lines = [f"{'cluster':>8}{'NoC cycles':>12}{'DRAM cycles':>13}{'speedup':>9}{'sweep min/mean/max':>22}"
+             f"{'NoC util':>10}{'HBM util NoC/DRAM':>19}"]
+    for r in rows:
+        lines.append(f"{r['cluster']:>8}{r['noc_makespan']:>12}{r['dram_makespan']:>13}{r['speedup']:>9.3f}"
+                     f"{r['speedup_min']:>10.3f}/{r['speedup_mean']:.3f}/{r['speedup_max']:.3f}"
+                     f"{100 * r['noc_util']:>9.1f}%{100 * r['hbm_util_noc']:>11.1f}/{100 * r['hbm_util_dram']:.1f}%")
+    return "\n".join(lines)
+
+
 def format_table(rows):
     lines = [f"{'organisation':<16}{'tile':<15}{'ablation':<11}{'makespan':>10}{'perf':>7}{'tensor':>8}"
              f"{'sweep min/mean/max':>22}"]
@@ -70,11 +116,16 @@ def format_table(rows):
 
 def main():
     ap = argparse.ArgumentParser()
+    ap.add_argument("--study", default="pipelines", choices=["pipelines", "noc"])
     ap.add_argument("--points-per-graph", type=int, default=1)
     ap.add_argument("--json", default=None)
     args = ap.parse_args()
-    rows = run_study(args.points_per_graph)
-    print(format_table(rows))
+    if args.study == "noc":
+        rows = run_noc_study(args.points_per_graph)
+        print(format_noc_table(rows))
+    else:
+        rows = run_study(args.points_per_graph)
+        print(format_table(rows))
     if args.json:
         with open(args.json, "w") as f:
             json.dump(rows, f, indent=1)

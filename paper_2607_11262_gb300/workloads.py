@@ -694,6 +694,12 @@ def workload(name: str, points: int | None = None, instances: int | None = None)
         p = pipelines.study_params(len(cases), 64)
         d = (f"GEMM+SiLU pipeline study: 4 organisations x {len(pipelines.TILES)} tiles x 4 ablations, "
              "10 waves on 1 SM; 64 points per graph (DRAM and tensor rate swept)")
+    elif name == "noc_fusion":
+        from . import clusters
+        g, cases = clusters.study_set()
+        p = clusters.study_params(cases, points_per_graph=32)
+        d = ("cluster-fused attention decode (H 4096, 32 heads, d 128, KV 1024), clusters of 2-16 CTAs, "
+             "NoC vs DRAM exchanges; 32 points per graph (NoC and DRAM rates swept)")
     else:
         raise KeyError(name)
     if points is not None:
@@ -702,4 +708,4 @@ def workload(name: str, points: int | None = None, instances: int | None = None)
 
 
 WORKLOADS = ("gemm512", "wsgemm8192", "fa_fwd", "decoder", "stress")
-STUDIES = ("pipelines",)
+STUDIES = ("pipelines", "noc_fusion")

@@ -96,3 +96,24 @@ def test_dsmem_without_noc_is_a_row_error():
     res = H.run_gpu(g, p)
     assert list(res["status"]) == [-3, 0]
     _check_all(g, p, res)
+
+
+def test_noc_fusion_workload_and_study():
+    from paper_2607_11262_gb300 import clusters, study
+    w = W.workload("noc_fusion")
+    res = H.run_gpu(w.graph, w.params)
+    assert np.all(res["status"] == 0)
+    sample = list(range(0, w.params.shape[0], 9))
+    refs = oracle_run.simulate_points(w.graph, w.params, sample)
+    for q in sample:
+        H.assert_point_equal(w.graph, w.params[q], res, q, refs[q])
+    rows = study.run_noc_study(points_per_graph=2)
+    graph, cases = clusters.study_set()
+    params = clusters.study_params(cases, points_per_graph=2)
+    for r in rows:
+        a = cases.index((r["cluster"], "noc"))
+        b = cases.index((r["cluster"], "dram"))
+        ra = oracle_run.simulate(graph, params[2 * a])
+        rb = oracle_run.simulate(graph, params[2 * b])
+        assert (r["noc_makespan"], r["dram_makespan"]) == (ra.makespan, rb.makespan)
+        assert r["speedup"] == pytest.approx(rb.makespan / ra.makespan, rel=1e-12)
