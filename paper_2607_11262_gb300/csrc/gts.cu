@@ -809,15 +809,26 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         const uint32_t rel = (ew.y & 1u) ? t : f;
         const bool to_next = mine && ew.x == nx;  // the stream's next node becomes the head right below
         bool to_head = false, cross = false;
-        if (mine && !to_next) {
-          const uint32_t wc = ew.y >> 8;
-          uint32_t tcs = NONE;
-          if (wc == myc) {
-            tcs = cs;
-          } else {
-            for (uint32_t jj = 0; jj < P.L.Scta; jj++)
-              if (P.cta(jj)[C_ID] == wc) { tcs = jj; break; }
+        const uint32_t wc = ew.y >> 8;
+        uint32_t tcs = (mine && !to_next && wc == myc) ? cs : NONE;
+        // successors in other CTAs: find each one's CTA slot, all lanes searching together
+        uint32_t xm = g.cross_cta ? __ballot_sync(FULL, mine && !to_next && wc != myc) : 0u;
+        while (xm) {
+          const int j = __ffs(xm) - 1;
+          xm &= xm - 1;
+          const uint32_t wcj = __shfl_sync(FULL, wc, j);
+          uint32_t found = NONE;
+          for (uint32_t b0 = 0; b0 < P.L.Scta; b0 += 32) {
+            const uint32_t jj = b0 + lane;
+            const uint32_t hit = __ballot_sync(FULL, jj < P.L.Scta && P.cta(jj)[C_ID] == wcj);
+            if (hit) {
+              found = b0 + __ffs(hit) - 1;
+              break;
+            }
           }
+          if (lane == j) tcs = found;
+        }
+        if (mine && !to_next) {
           if (tcs != NONE) {
             uint32_t *ts = P.slot(tcs * P.W + ((ew.y >> 1) & 127u));
             if ((ts[F_HID] & ID_MASK) == ew.x) {
