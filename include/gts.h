@@ -209,6 +209,55 @@ size_t gts_graph_workspace_bytes(uint32_t n_nodes, uint32_t n_edges, uint32_t n_
 gts_status gts_graph_create(const gts_graph_desc *desc, void *stream, gts_graph **out);
 gts_status gts_graph_destroy(gts_graph *graph);
 
+/*
+ * Template-shared graphs (Section 6.4 "Graph construction": the CTAs of a
+ * regular kernel run isomorphic tile graphs, so one physical CTA graph is
+ * stored once and every logical CTA refers to it).  T templates hold
+ * n_tpl_nodes nodes in total; template t owns nodes tpl_node_off[t] ..
+ * tpl_node_off[t+1]-1, with successor lists in CSR (tpl_row_ptr, tpl_col as an
+ * index into the same template's nodes, tpl_ekind).  Logical CTA c runs
+ * template cta_template[c]; its nodes get the next block of logical ids in CTA
+ * order (CTA-major), so node u of template t in CTA c has id
+ *   base_c + (u - tpl_node_off[t]),  base_c = sum over c' < c of |template of c'|.
+ * Edges stay inside a CTA.  Stacked sets: graph g owns CTAs graph_cta_off[g] ..
+ * graph_cta_off[g+1]-1 and the nodes of those CTAs.  n_nodes / n_edges are the
+ * logical totals (checked).  All arrays are DEVICE pointers owned by the caller.
+ * Contract (else GTS_ERR_INVALID_GRAPH): template edges go forward inside their
+ * template, type < 8, warp < warps_per_cta, ekind < 2, cta_template[c] < T,
+ * cta_kernel non-decreasing within each graph.
+ */
+typedef struct {
+  uint32_t n_templates, n_tpl_nodes, n_tpl_edges;
+  uint32_t n_nodes, n_edges, n_ctas, warps_per_cta, n_graphs;
+  const uint32_t *graph_cta_off;   /* [n_graphs+1]; NULL allowed when n_graphs == 1 */
+  const uint32_t *tpl_node_off;    /* [n_templates+1] */
+  const uint32_t *tpl_row_ptr;     /* [n_tpl_nodes+1] */
+  const uint32_t *tpl_col;         /* [n_tpl_edges] */
+  const uint8_t  *tpl_ekind;       /* [n_tpl_edges] GTS_EDGE_* */
+  const uint8_t  *tpl_type;        /* [n_tpl_nodes] */
+  const uint16_t *tpl_warp;        /* [n_tpl_nodes] */
+  const uint32_t *tpl_work;        /* [n_tpl_nodes] */
+  const uint32_t *tpl_lat_extra;   /* [n_tpl_nodes] */
+  const uint32_t *cta_template;    /* [n_ctas] */
+  const uint32_t *cta_kernel;      /* [n_ctas] */
+  void *workspace;                 /* device, >= gts_template_workspace_bytes(...) */
+  size_t workspace_bytes;
+} gts_template_desc;
+
+/* Device workspace of gts_graph_create_templated: the packed logical graph
+ * (as gts_graph_workspace_bytes) plus the expansion tables.  0 when a size is
+ * out of range. */
+size_t gts_template_workspace_bytes(uint32_t n_templates, uint32_t n_tpl_nodes, uint32_t n_nodes, uint32_t n_edges,
+                                    uint32_t n_ctas, uint32_t warps_per_cta, uint32_t n_graphs);
+
+/* Checks the templates and the CTA table on the host (they are copied there;
+ * the logical graph never is), then expands the logical graph on the device
+ * into desc->workspace, in the same packed form gts_graph_create builds from
+ * the expanded graph.  Waits for `stream`.  *out borrows desc->cta_kernel and
+ * desc->workspace.  Errors: INVALID_ARG, INVALID_GRAPH, UNSUPPORTED (in-degree),
+ * NOMEM (workspace), CUDA. */
+gts_status gts_graph_create_templated(const gts_template_desc *desc, void *stream, gts_graph **out);
+
 /* Registers a table of design points: d_params is [n_points][GTS_NPARAM]
  * int32 on the device, borrowed by *out.  Copies it to the host to size the
  * per-warp on-chip state of each row; waits for `stream`.  Rows that break the

@@ -959,6 +959,89 @@ struct gts_results {
   cudaStream_t stream;
 };
 
+namespace {
+
+// The library's handle over a packed workspace.
+gts_status make_handle(const WsLayout &wl, char *ws, uint64_t n, uint64_t m, uint64_t C, uint64_t W, uint64_t G,
+                       const std::vector<uint32_t> &noff, const std::vector<uint32_t> &coff, const uint32_t *d_kernel,
+                       uint32_t row_nodes, uint32_t row_ctas, uint32_t cross, uint32_t class_mask, gts_graph **out) {
+  gts_graph *g = new (std::nothrow) gts_graph();
+  if (!g) return fail(GTS_ERR_INVALID_ARG, "host allocation failed");
+  g->n = (uint32_t)n; g->m = (uint32_t)m; g->C = (uint32_t)C; g->W = (uint32_t)W; g->G = (uint32_t)G;
+  cudaGetDevice(&g->device);
+  g->node_off = noff;
+  g->cta_off = coff;
+  DevGraph &dg = g->dg;
+  dg.rec = (const uint4 *)(ws + wl.rec);
+  dg.rng = (const uint4 *)(ws + wl.rng);
+  dg.succ = (const uint2 *)(ws + wl.succ);
+  dg.stream_first = (const uint32_t *)(ws + wl.first);
+  dg.cta_cnt = (const uint32_t *)(ws + wl.cnt);
+  dg.cta_kernel = d_kernel;
+  dg.node_off = (const uint32_t *)(ws + wl.noff);
+  dg.cta_off = (const uint32_t *)(ws + wl.coff);
+  dg.W = (uint32_t)W;
+  dg.G = (uint32_t)G;
+  dg.row_nodes = row_nodes;
+  dg.row_ctas = row_ctas;
+  dg.cross_cta = cross;
+  dg.class_mask = class_mask;
+  *out = g;
+  return GTS_OK;
+}
+
+// Expansion tables of a template-shared graph, after the packed graph.
+struct TplLayout {
+  size_t base, ebase, indeg, next, first, total;
+};
+
+bool tpl_layout(uint64_t T, uint64_t TN, uint64_t n, uint64_t m, uint64_t C, uint64_t W, uint64_t G, WsLayout &w,
+                TplLayout &x) {
+  if (!ws_layout(n, m, C, W, G, w) || T < 1 || T > TN + 1 || TN >= 0x7FFFFFFEull) return false;
+  size_t o = w.total;
+  x.base = o; o += align_up(C * 4);
+  x.ebase = o; o += align_up(C * 4);
+  x.indeg = o; o += align_up(TN * 4);
+  x.next = o; o += align_up(TN * 4);
+  x.first = o; o += align_up(T * W * 4);
+  x.total = o;
+  return true;
+}
+
+// One block per logical CTA (grid-stride): copy its template's nodes and
+// edges into the packed arrays at the CTA's node and edge base, turning
+// template indices into logical ids.
+__global__ void k_expand(const uint32_t *__restrict__ cta_tpl, const uint32_t *__restrict__ tpl_off,
+                         const uint32_t *__restrict__ row_ptr, const uint32_t *__restrict__ col,
+                         const uint8_t *__restrict__ ek, const uint8_t *__restrict__ ty,
+                         const uint16_t *__restrict__ wp, const uint32_t *__restrict__ work,
+                         const uint32_t *__restrict__ lx, const uint32_t *__restrict__ cbase,
+                         const uint32_t *__restrict__ cebase, const uint32_t *__restrict__ tindeg,
+                         const uint32_t *__restrict__ tnext, const uint32_t *__restrict__ tfirst, uint32_t C, uint32_t W,
+                         uint4 *rec, uint4 *rng, uint2 *succ, uint32_t *first, uint32_t *cnt) {
+  for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
+    const uint32_t t = cta_tpl[c], u0 = tpl_off[t], u1 = tpl_off[t + 1];
+    const uint32_t base = cbase[c], eb = cebase[c], x0 = row_ptr[u0];
+    for (uint32_t u = u0 + threadIdx.x; u < u1; u += blockDim.x) {
+      const uint32_t v = base + (u - u0), nx = tnext[u];
+      rec[v] = make_uint4(work[u], lx[u], nx == NONE ? NONE : base + (nx - u0), (uint32_t)ty[u] | (tindeg[u] << 4));
+      const uint32_t a = row_ptr[u], b = row_ptr[u + 1];
+      rng[v] = make_uint4(0u, 0u, eb + (a - x0), eb + (b - x0));
+      for (uint32_t x = a; x < b; x++) {
+        const uint32_t w = col[x];
+        succ[eb + (x - x0)] = make_uint2(base + (w - u0), (uint32_t)ek[x] | ((uint32_t)wp[w] << 1) | (c << 8));
+      }
+    }
+    for (uint32_t w = threadIdx.x; w < W; w += blockDim.x) {
+      const uint32_t f = tfirst[(size_t)t * W + w];
+      first[(size_t)c * W + w] = f == NONE ? NONE : base + (f - u0);
+    }
+    if (threadIdx.x == 0) cnt[c] = u1 - u0;
+  }
+}
+
+}  // namespace
+
 extern "C" {
 
 const char *gts_last_error(void) { return g_err; }
@@ -1081,29 +1164,135 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "graph_create: copy to device");
 
-  gts_graph *g = new (std::nothrow) gts_graph();
-  if (!g) return fail(GTS_ERR_INVALID_ARG, "host allocation failed");
-  g->n = (uint32_t)n; g->m = (uint32_t)m; g->C = (uint32_t)C; g->W = (uint32_t)W; g->G = (uint32_t)G;
-  cudaGetDevice(&g->device);
-  g->node_off = noff;
-  g->cta_off = coff;
-  DevGraph &dg = g->dg;
-  dg.rec = (const uint4 *)(ws + wl.rec);
-  dg.rng = (const uint4 *)(ws + wl.rng);
-  dg.succ = (const uint2 *)(ws + wl.succ);
-  dg.stream_first = (const uint32_t *)(ws + wl.first);
-  dg.cta_cnt = (const uint32_t *)(ws + wl.cnt);
-  dg.cta_kernel = d->cta_kernel;
-  dg.node_off = (const uint32_t *)(ws + wl.noff);
-  dg.cta_off = (const uint32_t *)(ws + wl.coff);
-  dg.W = (uint32_t)W;
-  dg.G = (uint32_t)G;
-  dg.row_nodes = row_nodes;
-  dg.row_ctas = row_ctas;
-  dg.cross_cta = cross;
-  dg.class_mask = class_mask;
-  *out = g;
-  return GTS_OK;
+  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, cross, class_mask, out);
+}
+
+size_t gts_template_workspace_bytes(uint32_t n_templates, uint32_t n_tpl_nodes, uint32_t n_nodes, uint32_t n_edges,
+                                    uint32_t n_ctas, uint32_t warps_per_cta, uint32_t n_graphs) {
+  WsLayout w;
+  TplLayout x;
+  if (!tpl_layout(n_templates, n_tpl_nodes, n_nodes, n_edges, n_ctas, warps_per_cta, n_graphs, w, x)) return 0;
+  return x.total;
+}
+
+gts_status gts_graph_create_templated(const gts_template_desc *d, void *stream, gts_graph **out) {
+  clear_error();
+  if (!d || !out) return fail(GTS_ERR_INVALID_ARG, "null desc or out");
+  *out = nullptr;
+  const uint64_t T = d->n_templates, TN = d->n_tpl_nodes, TE = d->n_tpl_edges;
+  const uint64_t n = d->n_nodes, m = d->n_edges, C = d->n_ctas, W = d->warps_per_cta, G = d->n_graphs;
+  WsLayout wl;
+  TplLayout xl;
+  if (!tpl_layout(T, TN, n, m, C, W, G, wl, xl) || TE >= 0xFFFFFFFFull)
+    return fail(GTS_ERR_INVALID_ARG, "size out of range (1 <= templates, n < 2^31-1, C < 2^24, 1 <= W <= 128)");
+  if (!d->tpl_node_off || !d->tpl_row_ptr || (TN && (!d->tpl_type || !d->tpl_warp || !d->tpl_work || !d->tpl_lat_extra)) ||
+      (TE && (!d->tpl_col || !d->tpl_ekind)) || (C && (!d->cta_template || !d->cta_kernel)))
+    return fail(GTS_ERR_INVALID_ARG, "null template array");
+  if (G > 1 && !d->graph_cta_off) return fail(GTS_ERR_INVALID_ARG, "stacked set needs graph_cta_off");
+  if (!d->workspace) return fail(GTS_ERR_INVALID_ARG, "null workspace");
+  if (d->workspace_bytes < xl.total)
+    return fail(GTS_ERR_NOMEM, "workspace too small: need " + std::to_string(xl.total) + " bytes");
+  cudaStream_t s = (cudaStream_t)stream;
+  std::vector<uint32_t> toff, row_ptr, col, work, lx, ctpl, kern, coff;
+  std::vector<uint8_t> ek, ty;
+  std::vector<uint16_t> wp;
+  cudaError_t e = cudaSuccess;
+  if (e == cudaSuccess) e = d2h(toff, d->tpl_node_off, T + 1, s);
+  if (e == cudaSuccess) e = d2h(row_ptr, d->tpl_row_ptr, TN + 1, s);
+  if (e == cudaSuccess) e = d2h(col, d->tpl_col, TE, s);
+  if (e == cudaSuccess) e = d2h(ek, d->tpl_ekind, TE, s);
+  if (e == cudaSuccess) e = d2h(ty, d->tpl_type, TN, s);
+  if (e == cudaSuccess) e = d2h(wp, d->tpl_warp, TN, s);
+  if (e == cudaSuccess) e = d2h(work, d->tpl_work, TN, s);
+  if (e == cudaSuccess) e = d2h(lx, d->tpl_lat_extra, TN, s);
+  if (e == cudaSuccess) e = d2h(ctpl, d->cta_template, C, s);
+  if (e == cudaSuccess) e = d2h(kern, d->cta_kernel, C, s);
+  if (e == cudaSuccess) {
+    if (G > 1 || d->graph_cta_off) e = d2h(coff, d->graph_cta_off, G + 1, s);
+    else coff = {0u, (uint32_t)C};
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "graph_create_templated: copy to host");
+
+  // ---- contract on the templates
+  if (toff[0] != 0 || toff[T] != TN) return fail(GTS_ERR_INVALID_GRAPH, "tpl_node_off must run from 0 to n_tpl_nodes");
+  if (row_ptr[0] != 0 || row_ptr[TN] != TE) return fail(GTS_ERR_INVALID_GRAPH, "tpl_row_ptr must run from 0 to n_tpl_edges");
+  std::vector<uint32_t> tmask(T, 0u), tindeg(TN, 0u), tnext(TN, NONE), tfirst(T * W, NONE);
+  for (uint64_t t = 0; t < T; t++) {
+    if (toff[t + 1] < toff[t]) return fail(GTS_ERR_INVALID_GRAPH, "tpl_node_off decreases at template " + std::to_string(t));
+    const uint32_t u0 = toff[t], u1 = toff[t + 1];
+    for (uint32_t u = u0; u < u1; u++) {
+      if (row_ptr[u + 1] < row_ptr[u]) return fail(GTS_ERR_INVALID_GRAPH, "tpl_row_ptr decreases at node " + std::to_string(u));
+      if (ty[u] > GTS_DSMEM) return fail(GTS_ERR_INVALID_GRAPH, "bad type at template node " + std::to_string(u));
+      if (wp[u] >= W) return fail(GTS_ERR_INVALID_GRAPH, "warp >= warps_per_cta at template node " + std::to_string(u));
+      const uint32_t cls_v = (TYPE_CLASS >> (4 * ty[u])) & 15u;
+      if (cls_v < RC_N) tmask[t] |= 1u << cls_v;
+      if (cls_v == RC_DSM) tmask[t] |= (1u << RC_LSU) | CM_NOC;
+      for (uint32_t x = row_ptr[u]; x < row_ptr[u + 1]; x++) {
+        if (col[x] <= u || col[x] >= u1)
+          return fail(GTS_ERR_INVALID_GRAPH, "template edge " + std::to_string(x) + " must go forward inside its template");
+        if (ek[x] > 1) return fail(GTS_ERR_INVALID_GRAPH, "bad edge kind at template edge " + std::to_string(x));
+        if (++tindeg[col[x]] > MAX_INDEG)
+          return fail(GTS_ERR_UNSUPPORTED, "template node " + std::to_string(col[x]) + " has more than 2^24-1 predecessors");
+      }
+    }
+    for (uint32_t u = u1; u-- > u0;) {  // program order of each warp stream: ascending
+      tnext[u] = tfirst[t * W + wp[u]];
+      tfirst[t * W + wp[u]] = u;
+    }
+  }
+  // ---- the CTA table: node and edge bases (CTA-major), graph ranges
+  if (coff[0] != 0 || coff[G] != C) return fail(GTS_ERR_INVALID_GRAPH, "graph_cta_off must run from 0 to n_ctas");
+  std::vector<uint32_t> cbase(C), cebase(C), noff(G + 1);
+  uint64_t nb = 0, eb = 0;
+  uint32_t row_nodes = 0, row_ctas = 0, class_mask = 0;
+  for (uint64_t k = 0; k < G; k++) {
+    if (coff[k + 1] < coff[k]) return fail(GTS_ERR_INVALID_GRAPH, "graph_cta_off decreases at graph " + std::to_string(k));
+    noff[k] = (uint32_t)nb;
+    for (uint32_t c = coff[k]; c < coff[k + 1]; c++) {
+      const uint32_t t = ctpl[c];
+      if (t >= T) return fail(GTS_ERR_INVALID_GRAPH, "cta_template out of range at CTA " + std::to_string(c));
+      if (c > coff[k] && kern[c] < kern[c - 1])
+        return fail(GTS_ERR_INVALID_GRAPH, "cta_kernel decreases at CTA " + std::to_string(c));
+      cbase[c] = (uint32_t)nb;
+      cebase[c] = (uint32_t)eb;
+      nb += toff[t + 1] - toff[t];
+      eb += row_ptr[toff[t + 1]] - row_ptr[toff[t]];
+      class_mask |= tmask[t];
+      if (nb > n || eb > m) return fail(GTS_ERR_INVALID_GRAPH, "templates hold more nodes or edges than n_nodes / n_edges");
+    }
+    row_nodes = std::max(row_nodes, (uint32_t)(nb - noff[k]));
+    row_ctas = std::max(row_ctas, coff[k + 1] - coff[k]);
+  }
+  noff[G] = (uint32_t)nb;
+  if (nb != n || eb != m) return fail(GTS_ERR_INVALID_GRAPH, "n_nodes / n_edges differ from the templates' totals");
+
+  // ---- tables to the device, then the expansion
+  char *ws = (char *)d->workspace;
+  auto up = [&](size_t off, const void *src, size_t bytes) {
+    if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(ws + off, src, bytes, cudaMemcpyHostToDevice, s);
+  };
+  up(xl.base, cbase.data(), C * 4);
+  up(xl.ebase, cebase.data(), C * 4);
+  up(xl.indeg, tindeg.data(), TN * 4);
+  up(xl.next, tnext.data(), TN * 4);
+  up(xl.first, tfirst.data(), T * W * 4);
+  up(wl.noff, noff.data(), (G + 1) * 4);
+  up(wl.coff, coff.data(), (G + 1) * 4);
+  if (e == cudaSuccess && C) {
+    const uint32_t blocks = (uint32_t)std::min<uint64_t>(C, 65535);
+    k_expand<<<blocks, 256, 0, s>>>(d->cta_template, d->tpl_node_off, d->tpl_row_ptr, d->tpl_col, d->tpl_ekind,
+                                    d->tpl_type, d->tpl_warp, d->tpl_work, d->tpl_lat_extra,
+                                    (const uint32_t *)(ws + xl.base), (const uint32_t *)(ws + xl.ebase),
+                                    (const uint32_t *)(ws + xl.indeg), (const uint32_t *)(ws + xl.next),
+                                    (const uint32_t *)(ws + xl.first), (uint32_t)C, (uint32_t)W, (uint4 *)(ws + wl.rec),
+                                    (uint4 *)(ws + wl.rng), (uint2 *)(ws + wl.succ), (uint32_t *)(ws + wl.first),
+                                    (uint32_t *)(ws + wl.cnt));
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "graph_create_templated: expansion");
+  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, 0u, class_mask, out);
 }
 
 gts_status gts_graph_destroy(gts_graph *g) {

@@ -43,7 +43,8 @@ GTS_POLICY_LOWEST_ID, GTS_POLICY_GTO, GTS_POLICY_RR = 0, 1, 2
 
 GTS_STATIC_SCRATCH_BYTES = 32 << 20
 
-EXPORTS = ("gts_graph_workspace_bytes", "gts_graph_create", "gts_graph_destroy", "gts_params_upload",
+EXPORTS = ("gts_graph_workspace_bytes", "gts_graph_create", "gts_graph_destroy", "gts_template_workspace_bytes",
+           "gts_graph_create_templated", "gts_params_upload",
            "gts_params_destroy", "gts_row_nodes", "gts_row_ctas", "gts_scratch_bytes", "gts_simulate_batch",
            "gts_read_results", "gts_results_destroy", "gts_simulate_batch_noalloc", "gts_last_error")
 
@@ -61,6 +62,17 @@ class GraphDesc(ctypes.Structure):
                 ("row_ptr", ctypes.c_void_p), ("col", ctypes.c_void_p), ("ekind", ctypes.c_void_p),
                 ("type", ctypes.c_void_p), ("warp", ctypes.c_void_p), ("cta", ctypes.c_void_p),
                 ("work", ctypes.c_void_p), ("lat_extra", ctypes.c_void_p), ("cta_kernel", ctypes.c_void_p),
+                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t)]
+
+
+class TemplateDesc(ctypes.Structure):
+    _fields_ = [("n_templates", ctypes.c_uint32), ("n_tpl_nodes", ctypes.c_uint32), ("n_tpl_edges", ctypes.c_uint32),
+                ("n_nodes", ctypes.c_uint32), ("n_edges", ctypes.c_uint32), ("n_ctas", ctypes.c_uint32),
+                ("warps_per_cta", ctypes.c_uint32), ("n_graphs", ctypes.c_uint32),
+                ("graph_cta_off", ctypes.c_void_p), ("tpl_node_off", ctypes.c_void_p), ("tpl_row_ptr", ctypes.c_void_p),
+                ("tpl_col", ctypes.c_void_p), ("tpl_ekind", ctypes.c_void_p), ("tpl_type", ctypes.c_void_p),
+                ("tpl_warp", ctypes.c_void_p), ("tpl_work", ctypes.c_void_p), ("tpl_lat_extra", ctypes.c_void_p),
+                ("cta_template", ctypes.c_void_p), ("cta_kernel", ctypes.c_void_p),
                 ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t)]
 
 
@@ -83,6 +95,10 @@ def load():
     lib.gts_graph_create.restype = i32
     lib.gts_graph_destroy.argtypes = [vp]
     lib.gts_graph_destroy.restype = i32
+    lib.gts_template_workspace_bytes.argtypes = [u32, u32, u32, u32, u32, u32, u32]
+    lib.gts_template_workspace_bytes.restype = sz
+    lib.gts_graph_create_templated.argtypes = [ctypes.POINTER(TemplateDesc), vp, pp]
+    lib.gts_graph_create_templated.restype = i32
     lib.gts_params_upload.argtypes = [vp, vp, u32, vp, pp]
     lib.gts_params_upload.restype = i32
     lib.gts_params_destroy.argtypes = [vp]
@@ -125,6 +141,17 @@ def gts_graph_create(desc: GraphDesc, stream: int = 0):
 
 def gts_graph_destroy(graph):
     _check(load().gts_graph_destroy(graph))
+
+
+def gts_template_workspace_bytes(n_templates, n_tpl_nodes, n_nodes, n_edges, n_ctas, warps_per_cta, n_graphs):
+    return int(load().gts_template_workspace_bytes(n_templates, n_tpl_nodes, n_nodes, n_edges, n_ctas,
+                                                   warps_per_cta, n_graphs))
+
+
+def gts_graph_create_templated(desc: TemplateDesc, stream: int = 0):
+    h = ctypes.c_void_p()
+    _check(load().gts_graph_create_templated(ctypes.byref(desc), stream, ctypes.byref(h)))
+    return h.value
 
 
 def gts_params_upload(graph, d_params: int, n_points: int, stream: int = 0):
@@ -194,11 +221,24 @@ def _stream_handle(stream):
     return stream.cuda_stream
 
 
+def _to_device(a, dev):
+    import torch
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint32:
+        a = a.view(np.int32)
+    elif a.dtype == np.uint16:
+        a = a.view(np.int16)
+    return torch.from_numpy(a).to(dev)
+
+
 class DeviceGraph:
-    """A workloads.Graph resident on the GPU, validated and packed by libgts."""
+    """A workloads.Graph (or a template-shared workloads.TemplateSet) resident on
+    the GPU, validated and packed by libgts."""
 
     FIELDS = ("row_ptr", "col", "ekind", "type", "warp", "cta", "work", "lat_extra", "cta_kernel",
               "node_off", "cta_off")
+    TEMPLATE_FIELDS = ("tpl_node_off", "row_ptr", "col", "ekind", "type", "warp", "work", "lat_extra",
+                       "cta_template", "cta_kernel", "graph_cta_off")
 
     def __init__(self, graph, device="cuda", stream=None, tensors=None):
         """``tensors`` (optional): the graph's arrays already on the device,
@@ -206,14 +246,12 @@ class DeviceGraph:
         import torch
         self.graph = graph
         dev = torch.device(device)
+        if hasattr(graph, "tpl_node_off"):
+            self._create_templated(graph, dev, stream)
+            return
 
         def t(a):
-            a = np.ascontiguousarray(a)
-            if a.dtype == np.uint32:
-                a = a.view(np.int32)
-            elif a.dtype == np.uint16:
-                a = a.view(np.int16)
-            return torch.from_numpy(a).to(dev)
+            return _to_device(a, dev)
         if tensors is None:
             tensors = {k: t(getattr(graph, k)) for k in self.FIELDS}
         else:
@@ -224,7 +262,7 @@ class DeviceGraph:
         if nbytes == 0:
             raise GtsError(GTS_ERR_INVALID_ARG, "graph size out of range")
         with torch.cuda.stream(stream) if stream is not None else _null():
-            self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+            self.workspace = torch.zeros(nbytes, dtype=torch.uint8, device=dev)  # padding included
         T = self.tensors
         d = GraphDesc(n, m, C, W, G, T["node_off"].data_ptr(), T["cta_off"].data_ptr(), T["row_ptr"].data_ptr(),
                       T["col"].data_ptr(), T["ekind"].data_ptr(), T["type"].data_ptr(), T["warp"].data_ptr(),
@@ -232,6 +270,30 @@ class DeviceGraph:
                       T["cta_kernel"].data_ptr(), self.workspace.data_ptr(), nbytes)
         self.desc = d
         self.handle = gts_graph_create(d, _stream_handle(stream))
+        self.row_nodes = gts_row_nodes(self.handle)
+        self.row_ctas = gts_row_ctas(self.handle)
+
+    def _create_templated(self, ts, dev, stream):
+        import torch
+        self.tensors = T = {k: _to_device(getattr(ts, k), dev) for k in self.TEMPLATE_FIELDS}
+        TN, TE = int(ts.tpl_node_off[-1]), int(ts.col.shape[0])
+        # logical totals; an out-of-range template index is left for libgts to refuse
+        nsz, esz = ts.sizes()
+        ct = np.minimum(ts.cta_template.astype(np.int64), max(ts.n_templates - 1, 0))
+        n, m = (int(nsz[ct].sum()), int(esz[ct].sum())) if ts.n_templates else (0, 0)
+        C, W, G = ts.n_ctas, ts.warps_per_cta, ts.n_graphs
+        nbytes = gts_template_workspace_bytes(ts.n_templates, TN, n, m, C, W, G)
+        if nbytes == 0:
+            raise GtsError(GTS_ERR_INVALID_ARG, "template set size out of range")
+        with torch.cuda.stream(stream) if stream is not None else _null():
+            self.workspace = torch.zeros(nbytes, dtype=torch.uint8, device=dev)  # padding included
+        d = TemplateDesc(ts.n_templates, TN, TE, n, m, C, W, G, T["graph_cta_off"].data_ptr(),
+                         T["tpl_node_off"].data_ptr(), T["row_ptr"].data_ptr(), T["col"].data_ptr(),
+                         T["ekind"].data_ptr(), T["type"].data_ptr(), T["warp"].data_ptr(), T["work"].data_ptr(),
+                         T["lat_extra"].data_ptr(), T["cta_template"].data_ptr(), T["cta_kernel"].data_ptr(),
+                         self.workspace.data_ptr(), nbytes)
+        self.desc = d
+        self.handle = gts_graph_create_templated(d, _stream_handle(stream))
         self.row_nodes = gts_row_nodes(self.handle)
         self.row_ctas = gts_row_ctas(self.handle)
 

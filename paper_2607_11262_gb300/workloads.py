@@ -267,6 +267,107 @@ class CtaTemplate:
                 np.array(self.ek, np.uint8))
 
 
+@dataclasses.dataclass
+class TemplateSet:
+    """A template-shared graph (Section 6.4 "Graph construction"): physical CTA
+    graphs stored once, and per logical CTA the template it runs and its kernel.
+
+    Template t owns template nodes ``tpl_node_off[t]:tpl_node_off[t+1]``;
+    successors are CSR over template nodes (``col`` indexes template nodes of
+    the same template, sorted by source then target).  CTA c's nodes take the
+    next block of logical ids in CTA order.  A stacked set gives each graph g
+    the CTAs ``graph_cta_off[g]:graph_cta_off[g+1]``.
+    """
+    name: str
+    warps_per_cta: int
+    tpl_node_off: np.ndarray   # uint32 [T+1]
+    row_ptr: np.ndarray        # uint32 [TN+1]
+    col: np.ndarray            # uint32 [TE]
+    ekind: np.ndarray          # uint8  [TE]
+    type: np.ndarray           # uint8  [TN]
+    warp: np.ndarray           # uint16 [TN]
+    work: np.ndarray           # uint32 [TN]
+    lat_extra: np.ndarray      # uint32 [TN]
+    cta_template: np.ndarray   # uint32 [C]
+    cta_kernel: np.ndarray     # uint32 [C]
+    graph_cta_off: np.ndarray  # uint32 [G+1]
+
+    @property
+    def n_templates(self):
+        return int(self.tpl_node_off.shape[0] - 1)
+
+    @property
+    def n_ctas(self):
+        return int(self.cta_template.shape[0])
+
+    @property
+    def n_graphs(self):
+        return int(self.graph_cta_off.shape[0] - 1)
+
+    def sizes(self):
+        """Nodes and edges of each template."""
+        off = self.tpl_node_off.astype(np.int64)
+        return np.diff(off), np.diff(self.row_ptr.astype(np.int64)[off])
+
+    @property
+    def n_nodes(self):
+        return int(self.sizes()[0][self.cta_template].sum())
+
+    @property
+    def n_edges(self):
+        return int(self.sizes()[1][self.cta_template].sum())
+
+    def expand(self) -> Graph:
+        """The logical graph (every CTA's copy of its template, CTA-major ids)."""
+        off = self.tpl_node_off.astype(np.int64)
+        nsz, esz = self.sizes()
+        ct = self.cta_template.astype(np.int64)
+        cnt = nsz[ct]
+        base = np.zeros(len(ct) + 1, np.int64)
+        np.cumsum(cnt, out=base[1:])
+        n = int(base[-1])
+        # template node of every logical node, and its CTA
+        cta = np.repeat(np.arange(len(ct)), cnt)
+        u = off[ct][cta] + (np.arange(n) - base[:-1][cta])
+        rp = self.row_ptr.astype(np.int64)
+        deg = rp[u + 1] - rp[u]
+        src = np.repeat(np.arange(n), deg)
+        first_edge = np.repeat(rp[u], deg)
+        x = first_edge + (np.arange(src.shape[0]) - np.repeat(np.cumsum(deg) - deg, deg))
+        dst = base[:-1][cta[src]] + (self.col.astype(np.int64)[x] - off[ct[cta[src]]])
+        graphs = self.graph_cta_off.astype(np.int64)
+        return from_edges(self.name, self.warps_per_cta, self.type[u], self.warp[u], cta.astype(np.uint32),
+                          self.work[u], self.lat_extra[u], self.cta_kernel, src, dst, self.ekind[x],
+                          node_off=base[graphs].astype(np.uint32), cta_off=self.graph_cta_off)
+
+
+def template_set(name, warps_per_cta, templates, cta_template, cta_kernel, graph_cta_off=None) -> TemplateSet:
+    """CtaTemplates plus the per-CTA table as a TemplateSet."""
+    frozen = [t.frozen() for t in templates]
+    sizes = [len(f[0]) for f in frozen]
+    off = np.zeros(len(frozen) + 1, np.int64)
+    np.cumsum(sizes, out=off[1:])
+    rows, cols, kinds = [np.zeros(1, np.int64)], [], []
+    edges_so_far = 0
+    for i, (_t, _w, _wk, _x, es, ed, ek) in enumerate(frozen):
+        order = np.lexsort((ed, es))
+        es, ed, ek = es[order], ed[order], ek[order]
+        cnt = np.bincount(es, minlength=sizes[i])
+        rows.append(edges_so_far + np.cumsum(cnt))
+        cols.append(off[i] + ed)
+        kinds.append(ek)
+        edges_so_far += len(es)
+    cat = lambda parts, dt: np.concatenate(parts).astype(dt) if parts else np.zeros(0, dt)  # noqa: E731
+    C = len(cta_template)
+    return TemplateSet(
+        name=name, warps_per_cta=int(warps_per_cta), tpl_node_off=off.astype(np.uint32),
+        row_ptr=np.concatenate(rows).astype(np.uint32), col=cat(cols, np.uint32), ekind=cat(kinds, np.uint8),
+        type=cat([f[0] for f in frozen], np.uint8), warp=cat([f[1] for f in frozen], np.uint16),
+        work=cat([f[2] for f in frozen], np.uint32), lat_extra=cat([f[3] for f in frozen], np.uint32),
+        cta_template=np.asarray(cta_template, np.uint32), cta_kernel=np.asarray(cta_kernel, np.uint32),
+        graph_cta_off=np.array([0, C], np.uint32) if graph_cta_off is None else np.asarray(graph_cta_off, np.uint32))
+
+
 def assemble(name, warps_per_cta, templates, cta_template, cta_kernel) -> Graph:
     """Replicate CTA templates into one graph (vectorised; CTAs laid out in order).
 
@@ -479,13 +580,20 @@ def ew_cta(warps=4, loads=(131072,), ew_ops=262144, stores=(131072,)):
 
 
 # ---------------------------------------------------------------- the five workloads
-def gemm512() -> Graph:
+def _build(name, warps, templates, cta_template, cta_kernel, templated):
+    """The logical graph, or with ``templated`` the template-shared form."""
+    if templated:
+        return template_set(name, warps, templates, cta_template, cta_kernel)
+    return assemble(name, warps, templates, cta_template, cta_kernel)
+
+
+def gemm512(templated=False):
     """GEMM M=N=K=512 fp16, 128x128x64 CTA tiles (4x4 = 16 CTAs), 4 warps, 2-stage."""
     tpl = gemm_2stage_cta(ksteps=512 // 64)
-    return assemble("gemm512", 4, [tpl], np.zeros(16, np.int64), np.zeros(16, np.uint32))
+    return _build("gemm512", 4, [tpl], np.zeros(16, np.int64), np.zeros(16, np.uint32), templated)
 
 
-def ws_gemm(M=8192, N=8192, K=8192, num_ctas=132, name="wsgemm8192") -> Graph:
+def ws_gemm(M=8192, N=8192, K=8192, num_ctas=132, name="wsgemm8192", templated=False):
     """Warp-specialised persistent GEMM (bf16, 128x256x64 tiles).
 
     (M/128)*(N/256) output tiles over ``num_ctas`` persistent CTAs (tile t ->
@@ -496,24 +604,24 @@ def ws_gemm(M=8192, N=8192, K=8192, num_ctas=132, name="wsgemm8192") -> Graph:
     kinds = sorted(set(per.tolist()), reverse=True)
     tpls = [ws_gemm_cta(k, K // 64) for k in kinds]
     ct = np.array([kinds.index(x) for x in per], np.int64)
-    return assemble(name, 3, tpls, ct, np.zeros(num_ctas, np.uint32))
+    return _build(name, 3, tpls, ct, np.zeros(num_ctas, np.uint32), templated)
 
 
-def wsgemm8192(num_ctas=132) -> Graph:
+def wsgemm8192(num_ctas=132, templated=False):
     """M=N=K=8192: 2048 tiles over 132 persistent CTAs, 128 k-steps per tile."""
-    return ws_gemm(8192, 8192, 8192, num_ctas)
+    return ws_gemm(8192, 8192, 8192, num_ctas, templated=templated)
 
 
-def fa_fwd(batch=4, heads=32, seq=4096, head_dim=128, q_block=128, kv_block=128) -> Graph:
+def fa_fwd(batch=4, heads=32, seq=4096, head_dim=128, q_block=128, kv_block=128, templated=False):
     """FlashAttention forward, non-causal: one CTA per (batch, head, Q block)."""
     assert head_dim == 128
     nq = seq // q_block
     tpl = fa_fwd_cta(seq // kv_block)
     C = batch * heads * nq
-    return assemble("fa_fwd", 3, [tpl], np.zeros(C, np.int64), np.zeros(C, np.uint32))
+    return _build("fa_fwd", 3, [tpl], np.zeros(C, np.int64), np.zeros(C, np.uint32), templated)
 
 
-def decoder_layer(hidden=4096, heads=32, ffn=11008, tokens=16384, seq=2048) -> Graph:
+def decoder_layer(hidden=4096, heads=32, ffn=11008, tokens=16384, seq=2048, templated=False):
     """One Llama-style decoder layer for prefill of ``tokens`` tokens (fp16).
 
     Kernels in stream order (each a kernel-boundary gate for the next):
@@ -556,7 +664,7 @@ def decoder_layer(hidden=4096, heads=32, ffn=11008, tokens=16384, seq=2048) -> G
     add(ew_cta(loads=(2 * fb,), ew_ops=rows_w * ffn * 4, stores=(fb,)), ew_ctas, 6)
     gemm(hidden, ffn, 7)
     add(ew_cta(loads=(hb, hb), ew_ops=rows_w * hidden, stores=(hb,)), ew_ctas, 8)
-    return assemble("decoder", 4, tpls, np.array(cta_t), np.array(cta_k, np.uint32))
+    return _build("decoder", 4, tpls, np.array(cta_t), np.array(cta_k, np.uint32), templated)
 
 
 def random_layered_dag(seed, n_nodes=100_000, layers=64, fan_in=(1, 4), lat_log2=(2.0, 12.0),
@@ -657,30 +765,38 @@ class Workload:
     params: np.ndarray
 
 
-def workload(name: str, points: int | None = None, instances: int | None = None) -> Workload:
-    """One of the five named workloads (graph + parameter table).
+TEMPLATED = ("gemm512", "wsgemm8192", "wsgemm_small", "fa_fwd", "decoder")
+
+
+def workload(name: str, points: int | None = None, instances: int | None = None,
+             templated: bool = False) -> Workload:
+    """One of the named workloads (graph + parameter table).
 
     ``points`` truncates the parameter table (the rows are drawn for the full
-    size, so a prefix is the same rows); ``instances`` shrinks the stress set.
+    size, so a prefix is the same rows); ``instances`` shrinks the stress set;
+    ``templated`` returns the graph as a TemplateSet (the workloads in
+    TEMPLATED, whose CTAs run shared templates).
     """
+    if templated and name not in TEMPLATED:
+        raise ValueError(f"{name} has no template-shared form")
     if name == "gemm512":
-        g = gemm512()
+        g = gemm512(templated)
         p = sweep_params(SEED0 + 1, 64, [AX_SMS, AX_HBM, (P_MMA_LAT, 16, 64)], 2)
         d = "GEMM 512^3 fp16, 128x128x64 tiles, 4 warps, 2-stage; 64 points"
     elif name == "wsgemm8192":
-        g = wsgemm8192()
+        g = wsgemm8192(templated=templated)
         p = sweep_params(SEED0 + 2, 4096, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE], 1)
         d = "WS persistent GEMM 8192^3 bf16, 128x256x64, 1 producer + 2 consumer WGs, 4-stage ring, 132 CTAs; 4096 points"
     elif name == "wsgemm_small":
-        g = ws_gemm(2048, 2048, 1024, 132, "wsgemm_small")
+        g = ws_gemm(2048, 2048, 1024, 132, "wsgemm_small", templated=templated)
         p = sweep_params(SEED0 + 2, 4096, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE], 1)
         d = "WS GEMM 2048x2048x1024 (profiling-size case of the wsgemm8192 kernel shape); 4096 points"
     elif name == "fa_fwd":
-        g = fa_fwd()
+        g = fa_fwd(templated=templated)
         p = sweep_params(SEED0 + 3, 1024, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE, AX_ALU_RATE], 1)
         d = "FlashAttention fwd B4 H32 S4096 d128 fp16, non-causal; 1024 points"
     elif name == "decoder":
-        g = decoder_layer()
+        g = decoder_layer(templated=templated)
         p = sweep_params(SEED0 + 4, 512, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE, AX_ALU_RATE], 1)
         d = "Llama-style decoder layer prefill, hidden 4096, 32 heads, FFN 11008, 8x2048 tokens; 512 points"
     elif name == "stress":
