@@ -272,7 +272,9 @@ def main():
     # ---- e2e: host buffers through the C ABI, copies inside the timed region
     e2e = None
     if rank == 0 or ws > 1:
-        e2e = measure_e2e(g, w.params, gts, stream)
+        from paper_2607_11262_gb300 import workloads as W
+        templates = W.workload(args.workload, templated=True).graph if args.workload in W.TEMPLATED else None
+        e2e = measure_e2e(g, w.params, gts, stream, templates=templates)
 
     if rank != 0:
         if ws > 1:
@@ -311,18 +313,24 @@ def main():
         torch.distributed.destroy_process_group()
 
 
-def measure_e2e(graph, params, gts, stream, reps=2):
+def measure_e2e(graph, params, gts, stream, reps=2, templates=None):
     """Same metric through the public API from pinned host buffers: graph and
     parameter upload (host->device), graph packing, the batch, and the
-    device->host read of the per-point makespans and statuses, every step."""
+    device->host read of the per-point makespans and statuses, every step.
+    With ``templates`` (the same graph as a TemplateSet) the graph goes in
+    template-shared form: templates and the CTA table are uploaded and libgts
+    expands them on the device."""
     import torch
     P = int(params.shape[0])
     node_points = node_points_of(graph, params)
-    host = {k: torch.from_numpy(np.ascontiguousarray(getattr(graph, k)).view(
-        np.int32 if getattr(graph, k).dtype == np.uint32 else (np.int16 if getattr(graph, k).dtype == np.uint16
-                                                                else getattr(graph, k).dtype))).pin_memory()
-            for k in ("row_ptr", "col", "ekind", "type", "warp", "cta", "work", "lat_extra", "cta_kernel",
-                      "node_off", "cta_off")}
+    src = templates if templates is not None else graph
+    keys = gts.DeviceGraph.TEMPLATE_FIELDS if templates is not None else gts.DeviceGraph.FIELDS
+
+    def pinned(a):
+        a = np.ascontiguousarray(a)
+        a = a.view(np.int32 if a.dtype == np.uint32 else (np.int16 if a.dtype == np.uint16 else a.dtype))
+        return torch.from_numpy(a).pin_memory()
+    host = {k: pinned(getattr(src, k)) for k in keys}
     hp = torch.from_numpy(np.ascontiguousarray(params, np.int32).reshape(-1)).pin_memory()
     h_mk = torch.empty(P, dtype=torch.int32).pin_memory()
     h_st = torch.empty(P, dtype=torch.int32).pin_memory()
@@ -337,7 +345,7 @@ def measure_e2e(graph, params, gts, stream, reps=2):
         with torch.cuda.stream(stream):
             dt = {k: v.to(dev, non_blocking=True) for k, v in host.items()}
             dpar = hp.to(dev, non_blocking=True)
-            dg = gts.DeviceGraph.from_device_tensors(graph, dt, stream=stream)
+            dg = gts.DeviceGraph.from_device_tensors(src, dt, stream=stream)
             dpp = gts.DeviceParams.from_device_tensor(dg, dpar, P, stream=stream)
             out = gts.alloc_outputs(dg, P, flags)
             gts.simulate(dg, dpp, flags=flags, out=out, stream=stream)
@@ -348,7 +356,7 @@ def measure_e2e(graph, params, gts, stream, reps=2):
         del out, dpp, dg, dt, dpar
     t = min(times)
     return {"value": node_points / t, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-            "seconds_per_step": t}
+            "seconds_per_step": t, "graph_input": "template-shared" if templates is not None else "logical"}
 
 
 if __name__ == "__main__":

@@ -247,7 +247,7 @@ class DeviceGraph:
         self.graph = graph
         dev = torch.device(device)
         if hasattr(graph, "tpl_node_off"):
-            self._create_templated(graph, dev, stream)
+            self._create_templated(graph, dev, stream, tensors)
             return
 
         def t(a):
@@ -273,9 +273,13 @@ class DeviceGraph:
         self.row_nodes = gts_row_nodes(self.handle)
         self.row_ctas = gts_row_ctas(self.handle)
 
-    def _create_templated(self, ts, dev, stream):
+    def _create_templated(self, ts, dev, stream, tensors=None):
         import torch
-        self.tensors = T = {k: _to_device(getattr(ts, k), dev) for k in self.TEMPLATE_FIELDS}
+        if tensors is None:
+            tensors = {k: _to_device(getattr(ts, k), dev) for k in self.TEMPLATE_FIELDS}
+        else:
+            dev = next(iter(tensors.values())).device
+        self.tensors = T = tensors
         TN, TE = int(ts.tpl_node_off[-1]), int(ts.col.shape[0])
         # logical totals; an out-of-range template index is left for libgts to refuse
         nsz, esz = ts.sizes()
@@ -299,6 +303,7 @@ class DeviceGraph:
 
     @classmethod
     def from_device_tensors(cls, graph, tensors, stream=None):
+        """``tensors`` keyed like FIELDS, or like TEMPLATE_FIELDS for a TemplateSet."""
         return cls(graph, stream=stream, tensors=tensors)
 
     def close(self):
