@@ -132,6 +132,9 @@ def load_workload(name, rank, points, policy="lowest_id", subpartitions=4):
     if rank > 0 and name == "pipelines":
         from paper_2607_11262_gb300 import pipelines
         w.params = pipelines.study_params(w.graph.n_graphs, 64, seed=W.SEED0 + 6 + 100 * rank)
+    elif rank > 0 and name == "l2_gemm":
+        from paper_2607_11262_gb300 import l2gemm
+        w.params = l2gemm.study_params(w.graph.n_graphs, points_per_capacity=8, seed=W.SEED0 + 8 + 100 * rank)
     elif rank > 0 and name == "noc_fusion":
         from paper_2607_11262_gb300 import clusters
         w.params = clusters.study_params(clusters.study_cases(), points_per_graph=32, seed=W.SEED0 + 7 + 100 * rank)

@@ -111,8 +111,25 @@ typedef int32_t gts_status;
 #define GTS_P_CAP_NOC      24  /* NoC servers per SM group (1..32) */
 #define GTS_P_CLUSTER_SMS  25  /* SMs per NoC group: SM s is in group s / cluster_sms (1..32) */
 /* NoC fields 22..25 are all 0 (no NoC: a graph with DSMEM nodes is then GTS_ERR_INVALID_PARAMS
- * for that row) or noc_bpc >= 1, noc_lat >= 0, 1 <= cap_noc <= 32, 1 <= cluster_sms <= 32.
- * 26..31 reserved, must be 0 */
+ * for that row) or noc_bpc >= 1, noc_lat >= 0, 1 <= cap_noc <= 32, 1 <= cluster_sms <= 32. */
+#define GTS_P_L2_BYTES     26  /* L2 capacity in bytes; 0: no L2 model */
+#define GTS_P_L2_LAT       27  /* L2 latency, cycles */
+#define GTS_P_L2_BPC       28  /* L2 bytes per cycle per memory-side server */
+/* L2 fields 26..28 are all 0, or l2_bytes >= 1, l2_lat >= 0, l2_bpc >= 1.
+ * 29..31 reserved, must be 0.
+ *
+ * L2 model (Section 5.2: a fully associative LRU cache over tile-derived
+ * accesses).  With l2_bytes > 0, every design point keeps an LRU list of the
+ * tiles its LOAD and STORE nodes name (gts_graph_desc.tile), each entry sized
+ * by the bytes of its latest access, updated in issue order; after an access
+ * the least recently used tiles are dropped until the total is <= l2_bytes.
+ *  - LOAD whose tile is resident (hit): base tma_lat + l2_lat, holds a
+ *    memory-side server ceil(work / l2_bpc) cycles;
+ *  - any other LOAD (miss, or no tile): base tma_lat + l2_lat + dram_lat,
+ *    ceil(work / hbm_bpc) cycles;
+ *  - STORE: timing as without L2; its tile becomes the most recent entry.
+ * The memory-side servers are the cap_hbm servers ("HBM" below): hits and
+ * misses share them.  Without the L2 model a LOAD has base tma_lat + dram_lat. */
 
 /*
  * Issue policies (Section 5.3: ready nodes sit in per-subpartition queues
@@ -149,7 +166,7 @@ typedef int32_t gts_status;
  * busy_r / (servers_r * makespan), with servers_r = cap_r * num_sms for the
  * per-SM classes, cap_hbm for HBM and cap_noc * ceil(num_sms / cluster_sms)
  * for the NoC. */
-#define GTS_BUSY_CLASSES 7
+#define GTS_BUSY_CLASSES 9
 #define GTS_BUSY_TENSOR  0
 #define GTS_BUSY_TMA     1
 #define GTS_BUSY_LSU     2
@@ -157,6 +174,8 @@ typedef int32_t gts_status;
 #define GTS_BUSY_BAR     4
 #define GTS_BUSY_HBM     5
 #define GTS_BUSY_NOC     6
+#define GTS_BUSY_L2_HITS 7   /* not cycles: LOAD nodes that hit in L2 (L2 model only) */
+#define GTS_BUSY_L2_LOADS 8  /* not cycles: LOAD nodes that named a tile (L2 model only) */
 
 typedef struct gts_graph gts_graph;
 typedef struct gts_params gts_params;
@@ -192,6 +211,9 @@ typedef struct {
   const uint32_t *cta_kernel;       /* [n_ctas] */
   void *workspace;                  /* device, >= gts_graph_workspace_bytes(...) */
   size_t workspace_bytes;
+  const uint32_t *tile;             /* [n_nodes] tile a LOAD/STORE reads or writes, < n_tiles, or
+                                       0xFFFFFFFF (none); ignored on other types; NULL: no tiles */
+  uint32_t n_tiles;                 /* tile ids of each graph of the stack are < n_tiles */
 } gts_graph_desc;
 
 /* Bytes of device workspace gts_graph_create needs for a graph of this size

@@ -44,6 +44,14 @@
  *   CTA launch latency 0; times are int64 here and any finish above
  *   2^31-1 is reported as overflow.
  *
+ * L2 (optional, Section 5.2: a fully associative LRU cache over tile-derived
+ * accesses): LOAD and STORE nodes may name a tile; an LRU list of tiles, each
+ * sized by its latest access, is updated at every such issue and trimmed from
+ * the least recent end to l2_bytes.  A LOAD whose tile is in the list hits:
+ * base tma_lat + l2_lat and ceil(work / l2_bpc) cycles on a memory-side (HBM)
+ * server; every other LOAD pays tma_lat + l2_lat + dram_lat and
+ * ceil(work / hbm_bpc).  STORE timing is unchanged.
+ *
  * Busy server-cycles (optional output): for each resource class the sum of
  * the occupancies of the nodes served by it -- the cycles its servers were
  * held (Section 5.2).  Utilisation (Section 7.1 reports the tensor cores')
@@ -76,7 +84,7 @@ enum {
   PR_SMEM_BPC, PR_SMEM_LAT, PR_MMA_FMA_PC, PR_MMA_LAT, PR_ALU_OPS_PC, PR_ALU_LAT,
   PR_BAR_LAT, PR_CAP_TENSOR, PR_CAP_TMA, PR_CAP_LSU, PR_CAP_ALU, PR_CAP_BAR,
   PR_CAP_HBM, PR_GRAPH_INDEX, PR_ISSUE_POLICY, PR_SUBPARTITIONS, PR_NOC_BPC, PR_NOC_LAT, PR_CAP_NOC,
-  PR_CLUSTER_SMS, PR_COUNT = 32
+  PR_CLUSTER_SMS, PR_L2_BYTES, PR_L2_LAT, PR_L2_BPC, PR_COUNT = 32
 };
 enum { POL_LOWEST_ID = 0, POL_GTO = 1, POL_RR = 2 };
 
@@ -91,14 +99,15 @@ int oracle_simulate(
     const uint32_t *work, const uint32_t *lat_extra, const uint32_t *cta_kernel,
     const int32_t *prm,
     int64_t *start, int64_t *finish, int64_t *makespan, int32_t *cta_sm,
-    int64_t *busy /* [RC_COUNT + 2]: per-SM classes, HBM, NoC; may be NULL */)
+    int64_t *busy /* [RC_COUNT + 4]: per-SM classes, HBM, NoC, L2 load hits, tracked loads; may be NULL */,
+    const uint32_t *tile /* [n] tile of a LOAD/STORE or 0xFFFFFFFF; may be NULL */, int64_t n_tiles)
 {
   int64_t v, e, c, w, k, r;
   int status = OR_OK;
   if (n < 0 || m < 0 || n_ctas < 0 || W < 1 || !prm || !makespan) return OR_ERR_INVALID_ARG;
-  int64_t busy_acc[RC_COUNT + 2] = {0, 0, 0, 0, 0, 0, 0};
+  int64_t busy_acc[RC_COUNT + 4] = {0, 0, 0, 0, 0, 0, 0, 0, 0};
   if (busy)
-    for (r = 0; r < RC_COUNT + 2; r++) busy[r] = 0;
+    for (r = 0; r < RC_COUNT + 4; r++) busy[r] = 0;
 
   /* ---- parameter row (Table "GPU configurations" quantities) ---- */
   const int64_t num_sms = prm[PR_NUM_SMS], cps = prm[PR_CTAS_PER_SM];
@@ -127,8 +136,16 @@ int oracle_simulate(
   } else if (noc_bpc != 0 || prm[PR_NOC_LAT] != 0 || cap_noc != 0) {
     return OR_ERR_INVALID_PARAMS;
   }
-  for (k = PR_CLUSTER_SMS + 1; k < PR_COUNT; k++)
+  const int64_t l2_cap = prm[PR_L2_BYTES], l2_lat = prm[PR_L2_LAT], l2_bpc = prm[PR_L2_BPC];
+  const int l2on = l2_cap != 0;              /* the row models the L2 */
+  if (l2on) {
+    if (l2_cap < 1 || l2_lat < 0 || l2_bpc < 1) return OR_ERR_INVALID_PARAMS;
+  } else if (l2_lat != 0 || l2_bpc != 0) {
+    return OR_ERR_INVALID_PARAMS;
+  }
+  for (k = PR_L2_BPC + 1; k < PR_COUNT; k++)
     if (prm[k] != 0) return OR_ERR_INVALID_PARAMS;
+  if (n_tiles < 0 || (tile && n_tiles < 1)) return OR_ERR_INVALID_ARG;
   const int64_t ngrp = noc ? (num_sms + csms - 1) / csms : 1;  /* NoC groups */
   const int64_t per = cps * W;               /* warp slots per SM */
   const int64_t nq = num_sms * (nsub ? nsub : 1);
@@ -140,6 +157,8 @@ int oracle_simulate(
     if (type[v] >= OT_COUNT || (int64_t)warp[v] >= W || (int64_t)cta[v] >= n_ctas) return OR_ERR_INVALID_GRAPH;
     for (e = row_ptr[v]; e < (int64_t)row_ptr[v + 1]; e++)
       if ((int64_t)col[e] <= v || (int64_t)col[e] >= n || ekind[e] > 1) return OR_ERR_INVALID_GRAPH;
+    if (tile && tile[v] != 0xFFFFFFFFu && (type[v] == OT_LOAD || type[v] == OT_STORE) && (int64_t)tile[v] >= n_tiles)
+      return OR_ERR_INVALID_GRAPH;
   }
   for (c = 1; c < n_ctas; c++)
     if (cta_kernel[c] < cta_kernel[c - 1]) return OR_ERR_INVALID_GRAPH;
@@ -169,10 +188,14 @@ int oracle_simulate(
   int64_t *hsrv = calloc((size_t)cap_hbm, sizeof(int64_t));
   int64_t *nsrv = calloc((size_t)(ngrp * (noc ? cap_noc : 1)), sizeof(int64_t)); /* NoC servers per group */
   int64_t *nocc = malloc(sizeof(int64_t) * (size_t)(n ? n : 1));
+  const int64_t nt = tile ? n_tiles : 1;     /* L2 list over tiles: links, membership, entry bytes */
+  int64_t *l2_prev = malloc(sizeof(int64_t) * (size_t)nt), *l2_next = malloc(sizeof(int64_t) * (size_t)nt);
+  int64_t *l2_in = calloc((size_t)nt, sizeof(int64_t)), *l2_sz = calloc((size_t)nt, sizeof(int64_t));
+  int64_t l2_head = -1, l2_tail = -1, l2_used = 0;
   for (r = 0; r < RC_COUNT; r++) srv[r] = calloc((size_t)(num_sms * cap[r]), sizeof(int64_t));
   int nomem = !cls || !occ || !hocc || !lat || !npend || !rdy || !nxt || !head || !rem || !endt ||
               !sm_of || !res || !res_cnt || !hsrv || !slot_of || !sub_avail || !sub_last || !cand || !cand_key ||
-              !nsrv || !nocc;
+              !nsrv || !nocc || !l2_prev || !l2_next || !l2_in || !l2_sz;
   for (r = 0; r < RC_COUNT; r++) nomem |= !srv[r];
   if (nomem) { status = OR_ERR_NOMEM; goto out; }
 
@@ -304,7 +327,38 @@ int oracle_simulate(
         v = best;
         c = cta[v];
         const int64_t sm = sm_of[c];
-        const int64_t f = t + lat[v];
+        int64_t lv = lat[v], hv = hocc[v];
+        const int64_t tv = (tile && (type[v] == OT_LOAD || type[v] == OT_STORE) && tile[v] != 0xFFFFFFFFu)
+                               ? (int64_t)tile[v] : -1;
+        if (l2on && type[v] == OT_LOAD) {      /* hit or miss decides latency and memory-side occupancy */
+          const int hit = tv >= 0 && l2_in[tv];
+          hv = hit ? cdiv(work[v], l2_bpc) : cdiv(work[v], hbm_bpc);
+          lv = prm[PR_TMA_LAT] + l2_lat + (hit ? 0 : prm[PR_DRAM_LAT]) + (int64_t)lat_extra[v] +
+               (occ[v] > hv ? occ[v] : hv);
+          if (tv >= 0) { busy_acc[RC_COUNT + 3]++; if (hit) busy_acc[RC_COUNT + 2]++; }
+        }
+        if (l2on && tv >= 0) {                 /* the tile becomes the most recent entry */
+          if (l2_in[tv]) {
+            if (l2_prev[tv] >= 0) l2_next[l2_prev[tv]] = l2_next[tv]; else l2_head = l2_next[tv];
+            if (l2_next[tv] >= 0) l2_prev[l2_next[tv]] = l2_prev[tv]; else l2_tail = l2_prev[tv];
+            l2_used -= l2_sz[tv];
+          }
+          l2_prev[tv] = -1;
+          l2_next[tv] = l2_head;
+          if (l2_head >= 0) l2_prev[l2_head] = tv; else l2_tail = tv;
+          l2_head = tv;
+          l2_in[tv] = 1;
+          l2_sz[tv] = work[v];
+          l2_used += work[v];
+          while (l2_used > l2_cap) {           /* drop least recent entries */
+            const int64_t y = l2_tail;
+            l2_tail = l2_prev[y];
+            if (l2_tail >= 0) l2_next[l2_tail] = -1; else l2_head = -1;
+            l2_in[y] = 0;
+            l2_used -= l2_sz[y];
+          }
+        }
+        const int64_t f = t + lv;
         if (f > INT32_LIMIT) { status = OR_ERR_OVERFLOW; goto out; }
         start[v] = t;
         finish[v] = f;
@@ -315,7 +369,7 @@ int oracle_simulate(
         }
         if (f > mkspan) mkspan = f;
         if (cls[v] >= 0) busy_acc[cls[v]] += occ[v];
-        if (hocc[v] >= 0) busy_acc[RC_COUNT] += hocc[v];
+        if (hv >= 0) busy_acc[RC_COUNT] += hv;
         if (nocc[v] >= 0) busy_acc[RC_COUNT + 1] += nocc[v];
         if (cls[v] >= 0) { /* take any free server of the class on this SM */
           for (int64_t q = 0; q < cap[cls[v]]; q++) {
@@ -323,9 +377,9 @@ int oracle_simulate(
             if (*s <= t) { *s = t + occ[v]; break; }
           }
         }
-        if (hocc[v] >= 0) {
+        if (hv >= 0) {
           for (int64_t q = 0; q < cap_hbm; q++)
-            if (hsrv[q] <= t) { hsrv[q] = t + hocc[v]; break; }
+            if (hsrv[q] <= t) { hsrv[q] = t + hv; break; }
         }
         if (nocc[v] >= 0) { /* any free NoC server of the SM's group */
           for (int64_t q = 0; q < cap_noc; q++) {
@@ -373,12 +427,13 @@ int oracle_simulate(
   }
   *makespan = mkspan;
   if (busy)
-    for (r = 0; r < RC_COUNT + 2; r++) busy[r] = busy_acc[r];
+    for (r = 0; r < RC_COUNT + 4; r++) busy[r] = busy_acc[r];
 
 out:
   free(cls); free(occ); free(hocc); free(lat); free(npend); free(rdy); free(nxt); free(head);
   free(rem); free(endt); free(sm_of); free(res); free(res_cnt); free(hsrv);
   free(slot_of); free(sub_avail); free(sub_last); free(cand); free(cand_key); free(nsrv); free(nocc);
+  free(l2_prev); free(l2_next); free(l2_in); free(l2_sz);
   for (r = 0; r < RC_COUNT; r++) free(srv[r]);
   return status;
 }

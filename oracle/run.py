@@ -44,7 +44,7 @@ def _load():
             lib = ctypes.CDLL(build())
             p = ctypes.c_void_p
             i64 = ctypes.c_int64
-            lib.oracle_simulate.argtypes = [i64, i64, i64, i64] + [p] * 15
+            lib.oracle_simulate.argtypes = [i64, i64, i64, i64] + [p] * 16 + [i64]
             lib.oracle_simulate.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -57,7 +57,8 @@ class Result:
     start: np.ndarray    # int64 [n]
     finish: np.ndarray   # int64 [n]
     cta_sm: np.ndarray   # int32 [C]
-    busy: np.ndarray = None  # int64 [7]: busy server-cycles of TENSOR, TMA, LSU, ALU, BAR, HBM, NoC
+    busy: np.ndarray = None  # int64 [9]: busy server-cycles of TENSOR, TMA, LSU, ALU, BAR, HBM, NoC; L2 load hits,
+    #                          loads naming a tile
 
 
 def _ptr(a):
@@ -65,7 +66,7 @@ def _ptr(a):
 
 
 def simulate_arrays(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
-                    warps_per_cta, params) -> Result:
+                    warps_per_cta, params, tile=None, n_tiles=0) -> Result:
     """One design point on one graph given as plain arrays (graph-local ids)."""
     lib = _load()
     a = dict(row_ptr=np.ascontiguousarray(row_ptr, np.uint32), col=np.ascontiguousarray(col, np.uint32),
@@ -75,6 +76,7 @@ def simulate_arrays(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_
              cta_kernel=np.ascontiguousarray(cta_kernel, np.uint32))
     prm = np.ascontiguousarray(params, np.int32)
     assert prm.shape == (32,)
+    tl = None if tile is None else np.ascontiguousarray(tile, np.uint32)
     n = a["type"].shape[0]
     m = a["col"].shape[0]
     C = a["cta_kernel"].shape[0]
@@ -82,11 +84,12 @@ def simulate_arrays(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_
     finish = np.empty(max(n, 1), np.int64)
     cta_sm = np.empty(max(C, 1), np.int32)
     mk = ctypes.c_int64(0)
-    busy = np.zeros(7, np.int64)
+    busy = np.zeros(9, np.int64)
     st = lib.oracle_simulate(n, m, C, int(warps_per_cta), _ptr(a["row_ptr"]), _ptr(a["col"]), _ptr(a["ekind"]),
                              _ptr(a["type"]), _ptr(a["warp"]), _ptr(a["cta"]), _ptr(a["work"]),
                              _ptr(a["lat_extra"]), _ptr(a["cta_kernel"]), _ptr(prm), _ptr(start), _ptr(finish),
-                             ctypes.byref(mk), _ptr(cta_sm), _ptr(busy))
+                             ctypes.byref(mk), _ptr(cta_sm), _ptr(busy), None if tl is None else _ptr(tl),
+                             int(n_tiles))
     return Result(int(st), int(mk.value), start[:n], finish[:n], cta_sm[:C], busy)
 
 
@@ -101,7 +104,7 @@ def simulate(graph, params_row) -> Result:
             return Result(ERR_INVALID_PARAMS, 0, np.zeros(0, np.int64), np.zeros(0, np.int64), np.zeros(0, np.int32))
         g = graph.subgraph(gi)
     return simulate_arrays(g.row_ptr, g.col, g.ekind, g.type, g.warp, g.cta, g.work, g.lat_extra,
-                           g.cta_kernel, g.warps_per_cta, prm)
+                           g.cta_kernel, g.warps_per_cta, prm, g.tile, g.n_tiles)
 
 
 # ------------------------------------------------------------ process pool

@@ -12,7 +12,12 @@ purpose in everything but the definition:
   server free-time multiset the oracle keeps);
 * under the per-subpartition issue policies, a scheduler has issued at t when
   a node of its warp slots started at t, and the slot it issued from last is
-  that of its latest-started node (read off the schedule, no scheduler state).
+  that of its latest-started node (read off the schedule, no scheduler state);
+* the L2 keeps no cache state: a LOAD hits when its tile was accessed before
+  and survived every trim since, i.e. after each later access its bytes plus
+  the bytes (as of then) of the other tiles accessed since still fit in the
+  capacity -- the LRU stack-distance property (Mattson et al. 1970) for
+  entries of changing sizes, read off the log of accesses in issue order.
 
 Pure Python; only for graphs of a few dozen nodes with short latencies.
 """
@@ -50,11 +55,16 @@ def node_costs(ty, work, lat_extra, prm):
     return cls, occ, hocc, nocc, lat
 
 
+NO_TILE = 0xFFFFFFFF
+
+
 def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel, warps_per_cta, prm,
-             t_limit=None):
+             t_limit=None, tile=None, info=None):
     """Returns (status, makespan, start list, finish list, cta_sm list).
 
-    status: 0 ok, -6 a finish above 2^31-1, -8 no progress possible.
+    status: 0 ok, -6 a finish above 2^31-1, -8 no progress possible.  With a
+    dict ``info``, also fills info["hbm_occ"] (memory-side occupancy per node
+    as issued) and info["l2"] = [LOAD hits, LOADs naming a tile].
     """
     n = len(type_)
     C = len(cta_kernel)
@@ -65,6 +75,25 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     cap = {"tensor": prm[13], "tma": prm[14], "lsu": prm[15], "alu": prm[16], "bar": prm[17]}
     cap_hbm = prm[18]
     cap_noc, group = prm[24], prm[25]
+    l2_cap, l2_lat, l2_bpc = prm[26], prm[27], prm[28]
+    accesses = []          # (tile, bytes) of LOAD/STORE nodes naming a tile, in issue order
+    dyn = {}               # node -> (memory-side occupancy, latency) decided at issue
+    l2_count = [0, 0]
+
+    def tile_of(v):
+        if tile is None or int(type_[v]) not in (LOAD, STORE) or int(tile[v]) == NO_TILE:
+            return None
+        return int(tile[v])
+
+    def l2_hit(x):
+        last = [k for k, (y, _b) in enumerate(accesses) if y == x]
+        if not last:
+            return False
+        since, worst = {}, 0
+        for y, b in accesses[last[-1] + 1:]:
+            since[y] = b
+            worst = max(worst, sum(since.values()))
+        return worst + accesses[last[-1]][1] <= l2_cap
     costs = [node_costs(int(type_[v]), int(work[v]), int(lat_extra[v]), prm) for v in range(n)]
     preds = [[] for _ in range(n)]
     for u in range(n):
@@ -76,11 +105,16 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
     cta_slot = [-1] * C
     launched = [False] * C
     total_lat = sum(c[4] for c in costs)
+    if l2_cap:   # with the L2 a LOAD can take up to l2_lat + work cycles more
+        total_lat += sum(l2_lat + int(work[v]) for v in range(n) if int(type_[v]) == LOAD)
     if t_limit is None:   # every cycle without an issue lies under some node's latency or issue slot
         t_limit = total_lat + n + 2
 
     def finish(v):
-        return start[v] + costs[v][4]
+        return start[v] + (dyn[v][1] if v in dyn else costs[v][4])
+
+    def hocc_of(u):
+        return dyn[u][0] if u in dyn else costs[u][2]
 
     def retired(c, t):
         return launched[c] and all(start[v] is not None and finish(v) <= t for v in members[c])
@@ -99,8 +133,8 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
         return k
 
     def busy_hbm(t):
-        return sum(1 for u in range(n) if start[u] is not None and costs[u][2] is not None
-                   and start[u] <= t < start[u] + costs[u][2])
+        return sum(1 for u in range(n) if start[u] is not None and hocc_of(u) is not None
+                   and start[u] <= t < start[u] + hocc_of(u))
 
     def busy_noc(grp, t):
         return sum(1 for u in range(n) if start[u] is not None and costs[u][3] is not None
@@ -181,12 +215,27 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
                 cands = scheduler_picks(cands, t)
             if cands:
                 v = min(cands)
+                x = tile_of(v)
+                if l2_cap and int(type_[v]) == LOAD:
+                    hit = x is not None and l2_hit(x)
+                    w = int(work[v])
+                    ho = -(-w // (l2_bpc if hit else prm[2]))
+                    occ = costs[v][1]
+                    dyn[v] = (ho, prm[5] + l2_lat + (0 if hit else prm[3]) + int(lat_extra[v]) + max(occ, ho))
+                    if x is not None:
+                        l2_count[0] += hit
+                        l2_count[1] += 1
+                if l2_cap and x is not None:
+                    accesses.append((x, int(work[v])))
                 start[v] = t
                 if finish(v) > 2**31 - 1:
                     return -6, 0, start, [None] * n, cta_sm
                 changed = True
         if all(s is not None for s in start):
             fin = [finish(v) for v in range(n)]
+            if info is not None:
+                info["hbm_occ"] = [hocc_of(v) for v in range(n)]
+                info["l2"] = list(l2_count)
             return 0, max(fin, default=0), start, fin, cta_sm
         t += 1
         if t > t_limit:
@@ -196,15 +245,18 @@ def simulate(row_ptr, col, ekind, type_, warp, cta, work, lat_extra, cta_kernel,
 CLASS_ORDER = ("tensor", "tma", "lsu", "alu", "bar", "hbm", "noc")
 
 
-def busy_cycles(type_, work, lat_extra, prm, start, makespan):
+def busy_cycles(type_, work, lat_extra, prm, start, makespan, info=None):
     """Busy server-cycles of each class, measured on a finished schedule by
     sweeping every cycle t in [0, makespan) and counting the servers held at t
     (a node holds one server of its class on [start, start + occupancy), one
     HBM server on [start, start + HBM occupancy) and one NoC server on
     [start, start + NoC occupancy)).  Returned in the order TENSOR, TMA, LSU,
-    ALU, BAR, HBM, NoC."""
+    ALU, BAR, HBM, NoC, then the L2 counts of ``info`` (from ``simulate``;
+    its memory-side occupancies replace the static ones)."""
     prm = [int(x) for x in prm]
     costs = [node_costs(int(type_[v]), int(work[v]), int(lat_extra[v]), prm) for v in range(len(type_))]
+    if info is not None:
+        costs = [(c[0], c[1], info["hbm_occ"][v], c[3], c[4]) for v, c in enumerate(costs)]
     total = dict.fromkeys(CLASS_ORDER, 0)
     for t in range(makespan):
         for v, (cls, occ, hocc, nocc, _lat) in enumerate(costs):
@@ -214,10 +266,10 @@ def busy_cycles(type_, work, lat_extra, prm, start, makespan):
                 total["hbm"] += 1
             if nocc is not None and start[v] <= t < start[v] + nocc:
                 total["noc"] += 1
-    return [total[k] for k in CLASS_ORDER]
+    return [total[k] for k in CLASS_ORDER] + (list(info["l2"]) if info is not None else [0, 0])
 
 
 def simulate_graph(g, prm, **kw):
     """Same, for a single workloads.Graph."""
     return simulate(g.row_ptr, g.col, g.ekind, g.type, g.warp, g.cta, g.work, g.lat_extra, g.cta_kernel,
-                    g.warps_per_cta, prm, **kw)
+                    g.warps_per_cta, prm, tile=g.tile, **kw)

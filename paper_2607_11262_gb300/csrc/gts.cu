@@ -124,6 +124,7 @@ struct DevGraph {
   const uint32_t *node_off;    // [G+1]
   const uint32_t *cta_off;     // [G+1]
   uint32_t W, G, row_nodes, row_ctas, cross_cta;
+  uint32_t n_tiles;     // tile ids of LOAD/STORE nodes (rng.x = tile + 1; 0: none)
   uint32_t class_mask;  // bit r < 5: some node uses per-SM class r; CM_NOC: some node crosses the NoC
 };
 
@@ -132,9 +133,10 @@ struct DevGraph {
 // warp; CTA slot j lives on SM j / ctas_per_sm (SM-major, so the lowest free
 // slot is on the lowest SM with room).  Only min(num_sms*cps, C) CTA slots can
 // ever be occupied (a launch always takes the lowest free slot).
-constexpr uint32_t O_MAG = GTS_NPARAM;       // 6 x 2 words: division constants of the 5 rates and the NoC rate
-constexpr uint32_t O_BASE = GTS_NPARAM + 12; // 8 words: base latency per node type
-constexpr uint32_t O_DYN = GTS_NPARAM + 20;  // first per-point array
+constexpr uint32_t O_MAG = GTS_NPARAM;       // 7 x 2 words: division constants of the 5 rates, NoC and L2 rates
+constexpr uint32_t O_BASE = GTS_NPARAM + 14; // 8 words: base latency per node type, then LOAD hit / miss with L2
+constexpr uint32_t O_L2B = O_BASE + 8;
+constexpr uint32_t O_DYN = GTS_NPARAM + 24;  // first per-point array
 static_assert(O_MAG % 2 == 0, "division constants are 8-byte words");
 // slot record (5 words): id|HBM, rdy, pending<<8 | deg<<3 | class, next, successor begin
 constexpr uint32_t F_HID = 0, F_RDY = 1, F_META = 2, F_NXT = 3, F_SB = 4, SLOT_WORDS = 5;
@@ -179,7 +181,12 @@ __host__ __device__ inline int check_row(const int32_t *p, uint32_t G, uint32_t 
     return GTS_ERR_INVALID_PARAMS;
   }
   if ((class_mask & CM_NOC) && csms == 0) return GTS_ERR_INVALID_PARAMS;  // DSMEM nodes, no NoC
-  for (int i = GTS_P_CLUSTER_SMS + 1; i < GTS_NPARAM; i++)
+  if (p[GTS_P_L2_BYTES] != 0) {
+    if (p[GTS_P_L2_BYTES] < 1 || p[GTS_P_L2_LAT] < 0 || p[GTS_P_L2_BPC] < 1) return GTS_ERR_INVALID_PARAMS;
+  } else if (p[GTS_P_L2_LAT] != 0 || p[GTS_P_L2_BPC] != 0) {
+    return GTS_ERR_INVALID_PARAMS;
+  }
+  for (int i = GTS_P_L2_BPC + 1; i < GTS_NPARAM; i++)
     if (p[i] != 0) return GTS_ERR_INVALID_PARAMS;
   return GTS_OK;
 }
@@ -281,9 +288,11 @@ struct Pt {
 
 // Occupancies and latency of a node (Section 5.2 throughput model): per-SM
 // class, HBM and NoC occupancy; latency = base + lat_extra + the largest.
+// l2: 0 no L2 model, 1 LOAD missed, 2 LOAD hit (L2 model, Section 5.2).
 template <bool EXT>
 __device__ __forceinline__ void node_cost(const uint32_t *sp, uint32_t type, uint32_t work, uint32_t lx,
-                                          uint32_t &occ, uint32_t &hocc, uint32_t &nocc, uint64_t &lat) {
+                                          uint32_t &occ, uint32_t &hocc, uint32_t &nocc, uint64_t &lat,
+                                          uint32_t l2 = 0u) {
   const uint32_t rt = (TYPE_RATE >> (4 * type)) & 15u;
   occ = rt == 5u ? 1u : 0u;
   if (rt < 5u) occ = cdiv_c(work, sp[GTS_P_HBM_BPC + 2 * rt], *reinterpret_cast<const uint64_t *>(sp + O_MAG + 2 * rt));
@@ -291,7 +300,12 @@ __device__ __forceinline__ void node_cost(const uint32_t *sp, uint32_t type, uin
   if ((TYPE_HBM >> type) & 1u) hocc = cdiv_c(work, sp[GTS_P_HBM_BPC], *reinterpret_cast<const uint64_t *>(sp + O_MAG));
   nocc = 0u;
   if (EXT && type == GTS_DSMEM) nocc = cdiv_c(work, sp[GTS_P_NOC_BPC], *reinterpret_cast<const uint64_t *>(sp + O_MAG + 10));
-  lat = (uint64_t)sp[O_BASE + type] + lx + max(max(occ, hocc), nocc);
+  uint32_t base = sp[O_BASE + type];
+  if (EXT && l2 != 0u && type == GTS_LOAD) {  // a hit is served by L2, a miss goes through L2 to DRAM
+    if (l2 == 2u) hocc = cdiv_c(work, sp[GTS_P_L2_BPC], *reinterpret_cast<const uint64_t *>(sp + O_MAG + 12));
+    base = sp[O_L2B + (l2 == 2u ? 0u : 1u)];
+  }
+  lat = (uint64_t)base + lx + max(max(occ, hocc), nocc);
 }
 
 // Key of slot i computed at cycle t (>= t; INF if it cannot issue yet).
@@ -569,6 +583,35 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
   }
 }
 
+// One access of the L2 model's LRU list of a design point (Section 5.2): tile
+// x becomes the most recent entry, sized b; least recent entries are dropped
+// until the total is <= cap.  T[x] = {previous (more recent), next (less
+// recent), bytes, listed}; head / tail / used live in the calling lane.
+// Returns whether x was listed before the access (a hit).  One lane calls it.
+__device__ __forceinline__ uint32_t l2_access(uint4 *T, uint32_t x, uint32_t b, uint32_t &head, uint32_t &tail,
+                                              uint64_t &used, uint64_t cap) {
+  uint32_t *Tw = reinterpret_cast<uint32_t *>(T);
+  const uint4 e = T[x];
+  if (e.w) {  // unlink
+    if (e.x != NONE) Tw[4 * e.x + 1] = e.y; else head = e.y;
+    if (e.y != NONE) Tw[4 * e.y + 0] = e.x; else tail = e.x;
+    used -= e.z;
+  }
+  T[x] = make_uint4(NONE, head, b, 1u);
+  if (head != NONE) Tw[4 * head + 0] = x; else tail = x;
+  head = x;
+  used += b;
+  while (used > cap) {  // every entry dropped leaves used <= cap at the latest
+    const uint32_t y = tail;
+    const uint4 ey = T[y];
+    tail = ey.x;
+    if (tail != NONE) Tw[4 * tail + 1] = NONE; else head = NONE;
+    Tw[4 * y + 3] = 0u;
+    used -= ey.z;
+  }
+  return e.w;
+}
+
 // EXT: the kernel instance that also runs the per-subpartition issue policies
 // and the NoC of DSMEM nodes; the host launches the plain instance when no row
 // asks for a policy and the graph has no DSMEM node.
@@ -601,9 +644,10 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     P.c0 = g.cta_off[gi];
     P.c1 = g.cta_off[gi + 1];
     const uint32_t CG = P.c1 - P.c0;
+    const bool l2on = EXT && status == GTS_OK && prm[GTS_P_L2_BYTES] != 0;
     if (status == GTS_OK) {
       if (!make_layout(prm, CG, P.W, g.class_mask, P.L) || P.L.words > budget_words ||
-          (!EXT && (P.L.nsub || P.L.cap_noc)))
+          (!EXT && (P.L.nsub || P.L.cap_noc || prm[GTS_P_L2_BYTES] != 0)))
         status = GTS_ERR_UNSUPPORTED;
     }
     if (status != GTS_OK) {
@@ -620,7 +664,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     P.policy = (uint32_t)prm[GTS_P_ISSUE_POLICY];
     P.st = (flags & GTS_FULL_TRACE) ? d_start + (size_t)q * g.row_nodes : nullptr;
     P.fi = (flags & GTS_FULL_TRACE) ? d_finish + (size_t)q * g.row_nodes : nullptr;
-    P.scr = scratch + (size_t)gw * ((g.row_nodes + 1u) & ~1u);
+    P.scr = scratch + (size_t)gw * (((g.row_nodes + 1u) & ~1u) + 2u * g.n_tiles);
+    uint4 *l2t = reinterpret_cast<uint4 *>(P.scr + ((g.row_nodes + 1u) & ~1u));  // L2 list records per tile
     int32_t *cta_sm_row = (flags & GTS_WANT_CTA_SM) ? d_cta_sm + (size_t)q * g.row_ctas : nullptr;
 
     // ---- per-point constants and cleared state
@@ -639,6 +684,11 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       *reinterpret_cast<uint64_t *>(sp + O_MAG + 2 * lane) = div_const((uint32_t)prm[GTS_P_HBM_BPC + 2 * lane]);
     } else if (lane == (int)RC_N) {
       *reinterpret_cast<uint64_t *>(sp + O_MAG + 10) = div_const((uint32_t)prm[GTS_P_NOC_BPC]);
+    } else if (lane == (int)RC_N + 1) {
+      *reinterpret_cast<uint64_t *>(sp + O_MAG + 12) = div_const((uint32_t)prm[GTS_P_L2_BPC]);
+    } else if (lane == 30) {  // LOAD base with the L2 model: hit, miss
+      sp[O_L2B] = (uint32_t)prm[GTS_P_TMA_LAT] + (uint32_t)prm[GTS_P_L2_LAT];
+      sp[O_L2B + 1] = (uint32_t)prm[GTS_P_TMA_LAT] + (uint32_t)prm[GTS_P_L2_LAT] + (uint32_t)prm[GTS_P_DRAM_LAT];
     }
     if (lane < 8) {  // base latency per type: LOAD, SMEM, MMA, EW, STORE, BAR, NOP
       uint32_t bl = 0;
@@ -677,6 +727,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       const uint32_t nz = nG / 2;
       for (uint32_t k = lane; k < nz; k += 32) z[k] = make_uint4(0, 0, 0, 0);
       if ((nG & 1u) && lane == 0) P.scr[nG - 1] = make_uint2(0, 0);
+      if (l2on)
+        for (uint32_t k = lane; k < g.n_tiles; k += 32) l2t[k] = make_uint4(0, 0, 0, 0);
     }
     if (cta_sm_row)
       for (uint32_t c = lane; c < CG; c += 32) cta_sm_row[c] = -1;
@@ -693,7 +745,10 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     uint32_t issued = 0;
     int32_t mk = 0;
     uint64_t digest = 0;
-    uint64_t busy = 0;  // lane r < 5: server-cycles of per-SM class r; lane 5: HBM
+    uint64_t busy = 0;  // lane r < 5: server-cycles of per-SM class r; 5: HBM; 6: NoC; 7, 8: L2 hits, loads
+    uint32_t l2_head = NONE, l2_tail = NONE;  // the L2 list (lane 0)
+    uint64_t l2_used = 0;
+    const uint64_t l2_cap = l2on ? (uint64_t)prm[GTS_P_L2_BYTES] : 0ull;
     uint64_t b = INF64;  // this lane's best (effective cycle << 32 | id) over its SMs
     uint32_t bsl = 0;    // ... and its slot
     if (!launch_ctas<EXT>(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
@@ -727,6 +782,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       // one round of independent loads: the issued node's record, the next
       // head's record, range and counters, and the successor entries
       const uint4 rv = g.rec[v];
+      const uint32_t tkey = l2on ? g.rng[v].x : 0u;  // tile + 1 of the node (0: none)
       uint4 rn = make_uint4(0, 0, 0, 0), qn = rn;
       uint2 cn = make_uint2(0, 0);
       if (nx != NONE) {
@@ -740,7 +796,19 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       if ((uint32_t)lane < deg) ew = g.succ[sb + lane];
       uint32_t occ, hocc, nocc;
       uint64_t lat;
-      node_cost<EXT>(sp, rv.w & 15u, rv.x, rv.y, occ, hocc, nocc, lat);
+      uint32_t l2 = 0u;  // L2 model: 1 LOAD missed, 2 LOAD hit
+      if (EXT && l2on) {
+        const uint32_t ty = rv.w & 15u;
+        const bool mem = (ty == GTS_LOAD || ty == GTS_STORE) && tkey != 0u;
+        uint32_t hit = 0u;
+        if (lane == 0 && mem) hit = l2_access(l2t, tkey - 1u, rv.x, l2_head, l2_tail, l2_used, l2_cap);
+        hit = __shfl_sync(FULL, hit, 0);
+        if (ty == GTS_LOAD) {
+          l2 = hit ? 2u : 1u;
+          busy += ((uint32_t)lane == GTS_BUSY_L2_HITS && hit) || ((uint32_t)lane == GTS_BUSY_L2_LOADS && mem) ? 1u : 0u;
+        }
+      }
+      node_cost<EXT>(sp, rv.w & 15u, rv.x, rv.y, occ, hocc, nocc, lat, l2);
       const uint64_t f64 = (uint64_t)t + lat;
       if (f64 > 0x7FFFFFFFull) { status = GTS_ERR_OVERFLOW; break; }
       const uint32_t f = (uint32_t)f64;
@@ -949,7 +1017,7 @@ struct gts_params {
   const int32_t *d_params;
   uint32_t n_points;
   std::vector<uint32_t> words;  // per row: shared words, 0 if the row is invalid or too large
-  std::vector<uint8_t> sched;   // per row: asks for a per-subpartition issue policy
+  std::vector<uint8_t> sched;   // per row: asks for a per-subpartition issue policy or the L2 model
 };
 
 struct gts_results {
@@ -964,7 +1032,8 @@ namespace {
 // The library's handle over a packed workspace.
 gts_status make_handle(const WsLayout &wl, char *ws, uint64_t n, uint64_t m, uint64_t C, uint64_t W, uint64_t G,
                        const std::vector<uint32_t> &noff, const std::vector<uint32_t> &coff, const uint32_t *d_kernel,
-                       uint32_t row_nodes, uint32_t row_ctas, uint32_t cross, uint32_t class_mask, gts_graph **out) {
+                       uint32_t row_nodes, uint32_t row_ctas, uint32_t cross, uint32_t class_mask, uint32_t n_tiles,
+                       gts_graph **out) {
   gts_graph *g = new (std::nothrow) gts_graph();
   if (!g) return fail(GTS_ERR_INVALID_ARG, "host allocation failed");
   g->n = (uint32_t)n; g->m = (uint32_t)m; g->C = (uint32_t)C; g->W = (uint32_t)W; g->G = (uint32_t)G;
@@ -986,6 +1055,7 @@ gts_status make_handle(const WsLayout &wl, char *ws, uint64_t n, uint64_t m, uin
   dg.row_ctas = row_ctas;
   dg.cross_cta = cross;
   dg.class_mask = class_mask;
+  dg.n_tiles = n_tiles;
   *out = g;
   return GTS_OK;
 }
@@ -1073,10 +1143,13 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   if (d->workspace_bytes < wl.total)
     return fail(GTS_ERR_NOMEM, "workspace too small: need " + std::to_string(wl.total) + " bytes");
   cudaStream_t s = (cudaStream_t)stream;
-  std::vector<uint32_t> row_ptr, col, cta, work, lx, kern, noff, coff;
+  std::vector<uint32_t> row_ptr, col, cta, work, lx, kern, noff, coff, tile;
   std::vector<uint8_t> ek, ty;
   std::vector<uint16_t> wp;
   cudaError_t e = cudaSuccess;
+  if (d->tile && (d->n_tiles == 0 || d->n_tiles > (1u << 28)))
+    return fail(GTS_ERR_INVALID_ARG, "tiles need 1 <= n_tiles <= 2^28");
+  if (e == cudaSuccess && d->tile) e = d2h(tile, d->tile, n, s);
   if (e == cudaSuccess) e = d2h(row_ptr, d->row_ptr, n + 1, s);
   if (e == cudaSuccess) e = d2h(col, d->col, m, s);
   if (e == cudaSuccess) e = d2h(ek, d->ekind, m, s);
@@ -1117,6 +1190,8 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
       if (cls_v == RC_DSM) class_mask |= (1u << RC_LSU) | CM_NOC;
       if (wp[v] >= W) return fail(GTS_ERR_INVALID_GRAPH, "warp >= warps_per_cta at node " + std::to_string(v));
       if (cta[v] < c0 || cta[v] >= c1) return fail(GTS_ERR_INVALID_GRAPH, "cta outside its graph at node " + std::to_string(v));
+      if (d->tile && tile[v] != NONE && (ty[v] == GTS_LOAD || ty[v] == GTS_STORE) && tile[v] >= d->n_tiles)
+        return fail(GTS_ERR_INVALID_GRAPH, "tile >= n_tiles at node " + std::to_string(v));
       for (uint32_t x = row_ptr[v]; x < row_ptr[v + 1]; x++) {
         if (col[x] <= v || col[x] >= n1)
           return fail(GTS_ERR_INVALID_GRAPH, "edge " + std::to_string(x) + " must go forward inside its graph");
@@ -1143,7 +1218,8 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   std::vector<uint4> rec(n), rng(n);
   for (uint64_t v = 0; v < n; v++) {
     rec[v] = make_uint4(work[v], lx[v], nxt[v], (uint32_t)ty[v] | (indeg[v] << 4));
-    rng[v] = make_uint4(0u, 0u, row_ptr[v], row_ptr[v + 1]);
+    const bool tiled = d->tile && tile[v] != NONE && (ty[v] == GTS_LOAD || ty[v] == GTS_STORE);
+    rng[v] = make_uint4(tiled ? tile[v] + 1u : 0u, 0u, row_ptr[v], row_ptr[v + 1]);
   }
   std::vector<uint2> succ(m);
   for (uint64_t x = 0; x < m; x++)
@@ -1164,7 +1240,8 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "graph_create: copy to device");
 
-  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, cross, class_mask, out);
+  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, cross, class_mask,
+                     d->tile ? d->n_tiles : 0u, out);
 }
 
 size_t gts_template_workspace_bytes(uint32_t n_templates, uint32_t n_tpl_nodes, uint32_t n_nodes, uint32_t n_edges,
@@ -1292,7 +1369,7 @@ gts_status gts_graph_create_templated(const gts_template_desc *d, void *stream, 
   }
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "graph_create_templated: expansion");
-  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, 0u, class_mask, out);
+  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, 0u, class_mask, 0u, out);
 }
 
 gts_status gts_graph_destroy(gts_graph *g) {
@@ -1320,7 +1397,7 @@ gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_p
   for (uint32_t p = 0; p < n_points; p++) {
     const int32_t *row = h.data() + (size_t)p * GTS_NPARAM;
     if (check_row(row, g->G, g->dg.class_mask) != GTS_OK) continue;
-    P->sched[p] = row[GTS_P_ISSUE_POLICY] != GTS_POLICY_LOWEST_ID;
+    P->sched[p] = row[GTS_P_ISSUE_POLICY] != GTS_POLICY_LOWEST_ID || row[GTS_P_L2_BYTES] != 0;
     const uint32_t gi = (uint32_t)row[GTS_P_GRAPH_INDEX];
     Layout L;
     if (make_layout(row, g->cta_off[gi + 1] - g->cta_off[gi], g->W, g->dg.class_mask, L)) P->words[p] = L.words;
@@ -1337,11 +1414,14 @@ gts_status gts_params_destroy(gts_params *p) {
 namespace {
 // Per-warp scratch: one (released-predecessor count, max release cycle) pair
 // per node of the largest graph, rounded to 16 bytes.
-uint64_t scratch_row_bytes(const gts_graph *g) { return (((uint64_t)g->dg.row_nodes + 1) & ~1ull) * 8; }
+// ... plus, for a graph with tiles, one 16-byte L2 list record per tile.
+uint64_t scratch_row_bytes(const gts_graph *g) {
+  return (((uint64_t)g->dg.row_nodes + 1) & ~1ull) * 8 + 16ull * g->dg.n_tiles;
+}
 
 struct Plan {
   uint32_t words, wpb, smem, blocks, warps;
-  bool sched;  // launch the extended instance (issue policies, NoC)
+  bool sched;  // launch the extended instance (issue policies, NoC, L2)
 };
 
 gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, uint32_t np, uint32_t flags,

@@ -34,9 +34,10 @@ GTS_WANT_DIGEST = 2
 GTS_WANT_CTA_SM = 4
 GTS_WANT_BUSY = 8
 
-GTS_BUSY_CLASSES = 7
-GTS_BUSY_TENSOR, GTS_BUSY_TMA, GTS_BUSY_LSU, GTS_BUSY_ALU, GTS_BUSY_BAR, GTS_BUSY_HBM, GTS_BUSY_NOC = range(7)
-BUSY_NAMES = ("tensor", "tma", "lsu", "alu", "bar", "hbm", "noc")
+GTS_BUSY_CLASSES = 9
+(GTS_BUSY_TENSOR, GTS_BUSY_TMA, GTS_BUSY_LSU, GTS_BUSY_ALU, GTS_BUSY_BAR, GTS_BUSY_HBM, GTS_BUSY_NOC,
+ GTS_BUSY_L2_HITS, GTS_BUSY_L2_LOADS) = range(9)
+BUSY_NAMES = ("tensor", "tma", "lsu", "alu", "bar", "hbm", "noc", "l2_hits", "l2_loads")
 
 GTS_NPARAM = 32
 GTS_POLICY_LOWEST_ID, GTS_POLICY_GTO, GTS_POLICY_RR = 0, 1, 2
@@ -62,7 +63,8 @@ class GraphDesc(ctypes.Structure):
                 ("row_ptr", ctypes.c_void_p), ("col", ctypes.c_void_p), ("ekind", ctypes.c_void_p),
                 ("type", ctypes.c_void_p), ("warp", ctypes.c_void_p), ("cta", ctypes.c_void_p),
                 ("work", ctypes.c_void_p), ("lat_extra", ctypes.c_void_p), ("cta_kernel", ctypes.c_void_p),
-                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t)]
+                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+                ("tile", ctypes.c_void_p), ("n_tiles", ctypes.c_uint32)]
 
 
 class TemplateDesc(ctypes.Structure):
@@ -254,6 +256,8 @@ class DeviceGraph:
             return _to_device(a, dev)
         if tensors is None:
             tensors = {k: t(getattr(graph, k)) for k in self.FIELDS}
+            if getattr(graph, "tile", None) is not None:
+                tensors["tile"] = t(graph.tile)
         else:
             dev = next(iter(tensors.values())).device
         self.tensors = tensors
@@ -267,7 +271,8 @@ class DeviceGraph:
         d = GraphDesc(n, m, C, W, G, T["node_off"].data_ptr(), T["cta_off"].data_ptr(), T["row_ptr"].data_ptr(),
                       T["col"].data_ptr(), T["ekind"].data_ptr(), T["type"].data_ptr(), T["warp"].data_ptr(),
                       T["cta"].data_ptr(), T["work"].data_ptr(), T["lat_extra"].data_ptr(),
-                      T["cta_kernel"].data_ptr(), self.workspace.data_ptr(), nbytes)
+                      T["cta_kernel"].data_ptr(), self.workspace.data_ptr(), nbytes,
+                      T["tile"].data_ptr() if "tile" in T else None, int(getattr(graph, "n_tiles", 0) or 0))
         self.desc = d
         self.handle = gts_graph_create(d, _stream_handle(stream))
         self.row_nodes = gts_row_nodes(self.handle)
@@ -407,7 +412,9 @@ def utilisation(busy, makespan, params):
     """Per-class utilisation of each point from its busy server-cycles:
     busy_r / (servers_r * makespan), servers_r = cap_r * num_sms for the per-SM
     classes, cap_hbm for HBM and cap_noc * ceil(num_sms / cluster_sms) for the
-    NoC; 0 where the makespan is 0 or the row has no NoC.  numpy in, numpy out
+    NoC; 0 where the makespan is 0 or the row has no NoC.  The two L2 entries
+    are counts, not cycles: column GTS_BUSY_L2_HITS holds the hit rate (hits /
+    loads naming a tile) and GTS_BUSY_L2_LOADS 0.  numpy in, numpy out
     ([n_points][GTS_BUSY_CLASSES] float64)."""
     import numpy as np
     busy = np.asarray(busy, np.float64)
@@ -418,5 +425,8 @@ def utilisation(busy, makespan, params):
     servers[:, 5] = prm[:, 18]
     groups = np.where(prm[:, 25] > 0, -(-prm[:, 0] // np.maximum(prm[:, 25], 1)), 0)
     servers[:, 6] = prm[:, 24] * groups
-    den = servers * mk[:, None]
-    return np.divide(busy, den, out=np.zeros_like(busy), where=den > 0)
+    den = servers[:, :7] * mk[:, None]
+    out = np.zeros_like(busy)
+    np.divide(busy[:, :7], den, out=out[:, :7], where=den > 0)
+    np.divide(busy[:, 7], busy[:, 8], out=out[:, 7], where=busy[:, 8] > 0)
+    return out

@@ -1,6 +1,6 @@
 """Case studies on the GPU: software pipelining and the tile-graph ablation
-(Section 7.1 "Software Pipelining Impact"; Section 6.4 ablation), and
-NoC-enabled fusion (Section 7.2).
+(Section 7.1 "Software Pipelining Impact"; Section 6.4 ablation), NoC-enabled
+fusion (Section 7.2), and the L2 model (Section 5.2) under two tile orders.
 
 Every (organisation, tile, ablation) graph of ``pipelines.study_set`` runs on
 one simulated Hopper SM through libgts; the table reports, per graph, the
@@ -14,7 +14,10 @@ The NoC study runs the cluster-fused attention decode of ``clusters`` with
 NoC and with DRAM exchanges for every cluster size and reports both makespans,
 the speedup and the NoC utilisation (busy NoC cycles / (servers x makespan)).
 
-    python -m paper_2607_11262_gb300.study [--study pipelines|noc] [--points-per-graph 64] [--json out.json]
+The L2 study runs the persistent GEMM of ``l2gemm`` in row-major and grouped
+rasterization at L2 capacities of 0-100 MB and reports makespan and hit rate.
+
+    python -m paper_2607_11262_gb300.study [--study pipelines|noc|l2] [--points-per-graph 64] [--json out.json]
 """
 from __future__ import annotations
 
@@ -23,7 +26,7 @@ import json
 
 import numpy as np
 
-from . import clusters, gts, pipelines
+from . import clusters, gts, l2gemm, pipelines
 
 
 def run_study(points_per_graph=1, device="cuda"):
@@ -93,6 +96,40 @@ def run_noc_study(points_per_graph=1, device="cuda"):
     return rows
 
 
+def run_l2_study(device="cuda"):
+    """L2 capacity x tile order; one dict per (order, capacity)."""
+    import torch
+    gts.load()
+    graph, orders = l2gemm.study_set()
+    params = l2gemm.study_params(len(orders))
+    dg = gts.DeviceGraph(graph, device=device)
+    dp = gts.DeviceParams(dg, params)
+    out = gts.simulate(dg, dp, flags=gts.GTS_WANT_BUSY)
+    torch.cuda.synchronize()
+    status = out.status.cpu().numpy()
+    if np.any(status != gts.GTS_OK):
+        raise gts.GtsError(int(status[status != 0][0]), "a study point did not simulate")
+    mk = out.makespan.cpu().numpy()
+    busy = out.busy.cpu().numpy()
+    dp.close()
+    dg.close()
+    rows = []
+    for q in range(params.shape[0]):
+        loads = int(busy[q, gts.GTS_BUSY_L2_LOADS])
+        rows.append(dict(order=orders[int(params[q, 19])], l2_mb=int(params[q, 26]) >> 20, makespan=int(mk[q]),
+                         hits=int(busy[q, gts.GTS_BUSY_L2_HITS]), loads=loads,
+                         hit_rate=float(busy[q, gts.GTS_BUSY_L2_HITS]) / loads if loads else 0.0))
+    return rows
+
+
+def format_l2_table(rows):
+    lines = [f"{'order':<10}{'L2 MB':>7}{'cycles':>12}{'hits':>9}{'loads':>9}{'hit rate':>10}"]
+    for r in rows:
+        lines.append(f"{r['order']:<10}{r['l2_mb']:>7}{r['makespan']:>12}{r['hits']:>9}{r['loads']:>9}"
+                     f"{100 * r['hit_rate']:>9.1f}%")
+    return "\n".join(lines)
+
+
 def format_noc_table(rows):
     lines = [f"{'cluster':>8}{'NoC cycles':>12}{'DRAM cycles':>13}{'speedup':>9}{'sweep min/mean/max':>22}"
              f"{'NoC util':>10}{'HBM util NoC/DRAM':>19}"]
@@ -116,13 +153,16 @@ def format_table(rows):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--study", default="pipelines", choices=["pipelines", "noc"])
+    ap.add_argument("--study", default="pipelines", choices=["pipelines", "noc", "l2"])
     ap.add_argument("--points-per-graph", type=int, default=1)
     ap.add_argument("--json", default=None)
     args = ap.parse_args()
     if args.study == "noc":
         rows = run_noc_study(args.points_per_graph)
         print(format_noc_table(rows))
+    elif args.study == "l2":
+        rows = run_l2_study()
+        print(format_l2_table(rows))
     else:
         rows = run_study(args.points_per_graph)
         print(format_table(rows))

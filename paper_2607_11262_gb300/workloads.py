@@ -43,13 +43,13 @@ NPARAM = 32
  P_SMEM_BPC, P_SMEM_LAT, P_MMA_FMA_PC, P_MMA_LAT, P_ALU_OPS_PC, P_ALU_LAT,
  P_BAR_LAT, P_CAP_TENSOR, P_CAP_TMA, P_CAP_LSU, P_CAP_ALU, P_CAP_BAR,
  P_CAP_HBM, P_GRAPH_INDEX, P_ISSUE_POLICY, P_SUBPARTITIONS, P_NOC_BPC, P_NOC_LAT, P_CAP_NOC,
- P_CLUSTER_SMS) = range(26)
+ P_CLUSTER_SMS, P_L2_BYTES, P_L2_LAT, P_L2_BPC) = range(29)
 PARAM_NAMES = ("num_sms", "ctas_per_sm", "hbm_bpc", "dram_lat", "tma_bpc",
                "tma_lat", "smem_bpc", "smem_lat", "mma_fma_pc", "mma_lat",
                "alu_ops_pc", "alu_lat", "bar_lat", "cap_tensor", "cap_tma",
                "cap_lsu", "cap_alu", "cap_bar", "cap_hbm", "graph_index",
                "issue_policy", "subpartitions", "noc_bpc", "noc_lat", "cap_noc",
-               "cluster_sms") + tuple(f"reserved{i}" for i in range(26, NPARAM))
+               "cluster_sms", "l2_bytes", "l2_lat", "l2_bpc") + tuple(f"reserved{i}" for i in range(29, NPARAM))
 # issue policies (Section 5.3): one global lowest-id order, or per-subpartition
 # greedy-then-oldest / round-robin schedulers issuing one node per cycle
 POLICY_LOWEST_ID, POLICY_GTO, POLICY_RR = 0, 1, 2
@@ -129,6 +129,8 @@ class Graph:
     cta_kernel: np.ndarray   # uint32 [C]
     node_off: np.ndarray     # uint32 [G+1]
     cta_off: np.ndarray      # uint32 [G+1]
+    tile: np.ndarray = None  # uint32 [n] tile a LOAD/STORE reads or writes (NO_TILE: none); None: no tiles
+    n_tiles: int = 0         # tile ids are < n_tiles
 
     @property
     def n_nodes(self) -> int:
@@ -164,7 +166,8 @@ class Graph:
             work=self.work[n0:n1].copy(), lat_extra=self.lat_extra[n0:n1].copy(),
             cta_kernel=self.cta_kernel[c0:c1].copy(),
             node_off=np.array([0, n1 - n0], np.uint32),
-            cta_off=np.array([0, c1 - c0], np.uint32))
+            cta_off=np.array([0, c1 - c0], np.uint32),
+            tile=None if self.tile is None else self.tile[n0:n1].copy(), n_tiles=self.n_tiles)
 
     def arrays(self):
         return {f.name: getattr(self, f.name) for f in dataclasses.fields(self)
@@ -176,11 +179,15 @@ class Graph:
             h.update(k.encode())
             h.update(np.ascontiguousarray(a).tobytes())
         h.update(str(self.warps_per_cta).encode())
+        h.update(str(self.n_tiles).encode())
         return h.hexdigest()
 
 
+NO_TILE = 0xFFFFFFFF
+
+
 def from_edges(name, warps_per_cta, type_, warp, cta, work, lat_extra, cta_kernel,
-               src, dst, kind, node_off=None, cta_off=None) -> Graph:
+               src, dst, kind, node_off=None, cta_off=None, tile=None, n_tiles=0) -> Graph:
     """Build a Graph from an edge list (sorted into CSR by source, then target)."""
     n = int(len(type_))
     src = np.asarray(src, np.int64)
@@ -201,7 +208,8 @@ def from_edges(name, warps_per_cta, type_, warp, cta, work, lat_extra, cta_kerne
                  warp=np.asarray(warp, np.uint16), cta=np.asarray(cta, np.uint32),
                  work=np.asarray(work, np.uint32), lat_extra=np.asarray(lat_extra, np.uint32),
                  cta_kernel=np.asarray(cta_kernel, np.uint32),
-                 node_off=np.asarray(node_off, np.uint32), cta_off=np.asarray(cta_off, np.uint32))
+                 node_off=np.asarray(node_off, np.uint32), cta_off=np.asarray(cta_off, np.uint32),
+                 tile=None if tile is None else np.asarray(tile, np.uint32), n_tiles=int(n_tiles))
 
 
 def stack(graphs, name) -> Graph:
@@ -226,7 +234,10 @@ def stack(graphs, name) -> Graph:
         work=np.concatenate([g.work for g in graphs]),
         lat_extra=np.concatenate([g.lat_extra for g in graphs]),
         cta_kernel=np.concatenate([g.cta_kernel for g in graphs]),
-        node_off=noff.astype(np.uint32), cta_off=coff.astype(np.uint32))
+        node_off=noff.astype(np.uint32), cta_off=coff.astype(np.uint32),
+        tile=(None if all(g.tile is None for g in graphs) else np.concatenate(
+            [g.tile if g.tile is not None else np.full(g.n_nodes, NO_TILE, np.uint32) for g in graphs])),
+        n_tiles=max(g.n_tiles for g in graphs))
 
 
 # ---------------------------------------------------------------- CTA templates
@@ -810,6 +821,12 @@ def workload(name: str, points: int | None = None, instances: int | None = None,
         p = pipelines.study_params(len(cases), 64)
         d = (f"GEMM+SiLU pipeline study: 4 organisations x {len(pipelines.TILES)} tiles x 4 ablations, "
              "10 waves on 1 SM; 64 points per graph (DRAM and tensor rate swept)")
+    elif name == "l2_gemm":
+        from . import l2gemm
+        g, orders = l2gemm.study_set()
+        p = l2gemm.study_params(len(orders), points_per_capacity=8)
+        d = ("persistent WS GEMM 4096^3 bf16, 128x256x64, 132 CTAs, A/B/C loads and stores naming tiles, row-major "
+             "and grouped rasterization; L2 0-100 MB (LRU over tiles), 8 DRAM rates each")
     elif name == "noc_fusion":
         from . import clusters
         g, cases = clusters.study_set()
@@ -824,4 +841,4 @@ def workload(name: str, points: int | None = None, instances: int | None = None,
 
 
 WORKLOADS = ("gemm512", "wsgemm8192", "fa_fwd", "decoder", "stress")
-STUDIES = ("pipelines", "noc_fusion")
+STUDIES = ("pipelines", "noc_fusion", "l2_gemm")

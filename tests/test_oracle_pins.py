@@ -147,6 +147,97 @@ def test_noc_parameter_checks():
         assert run.simulate(h, prm).status == run.ERR_INVALID_PARAMS, fields
 
 
+def _l2_graph(case_nodes):
+    n = len(case_nodes)
+    g = TG.make(n, [(v, v + 1, W.DATA) for v in range(n - 1)], [TYPE[x[0]] for x in case_nodes], [0] * n,
+                [0] * n, 1, work=[x[2] for x in case_nodes])
+    g.tile = np.array([W.NO_TILE if x[1] < 0 else x[1] for x in case_nodes], np.uint32)
+    g.n_tiles = 8
+    return g
+
+
+def _l2_params(l2_bytes, l2_lat=3, l2_bpc=2):
+    prm = TG.unit_params(1, 1)
+    prm[W.P_DRAM_LAT] = 10
+    prm[W.P_L2_BYTES], prm[W.P_L2_LAT], prm[W.P_L2_BPC] = l2_bytes, l2_lat, l2_bpc
+    return prm
+
+
+def test_golden_l2():
+    spec = json.load(open(os.path.join(GOLDEN, "l2.json")))
+    for case in spec["cases"]:
+        g = _l2_graph(case["nodes"])
+        prm = _l2_params(case["l2_bytes"])
+        r = run.simulate(g, prm)
+        assert r.status == 0, case["name"]
+        assert list(r.start) == case["start"], (case["name"], list(r.start))
+        assert list(r.finish) == case["finish"], (case["name"], list(r.finish))
+        assert (r.busy[7], r.busy[8], r.busy[5]) == (case["hits"], case["loads"], case["hbm_busy"]), case["name"]
+        info = {}
+        st, mk, start, fin, _ = stepper.simulate_graph(g, prm, info=info)
+        assert (st, list(r.start), list(r.finish)) == (0, start, fin)
+        assert list(r.busy) == stepper.busy_cycles(g.type, g.work, g.lat_extra, prm, start, mk, info)
+
+
+def test_stepper_equals_oracle_l2():
+    # the stepper decides hits by stack distance over its log of accesses, the
+    # oracle by an explicit LRU list
+    rng = np.random.default_rng(80)
+    types = (W.LOAD, W.LOAD, W.LOAD, W.STORE, W.MMA, W.EW, W.NOP)
+    for i in range(150):
+        n = int(rng.integers(2, 24))
+        g = TG.random_graph(rng, n, p_edge=float(rng.uniform(0.05, 0.35)), cta_major=bool(i % 3),
+                            kernels=bool(i % 5 == 0), types=types, max_work=9)
+        nt = int(rng.integers(1, 6))
+        t = rng.integers(0, nt, n).astype(np.uint32)
+        t[rng.random(n) < 0.15] = W.NO_TILE
+        g.tile, g.n_tiles = t, nt
+        prm = TG.small_params(rng)
+        prm[W.P_L2_BYTES] = int(rng.integers(1, 30))
+        prm[W.P_L2_LAT] = int(rng.integers(0, 5))
+        prm[W.P_L2_BPC] = int(rng.integers(1, 6))
+        if i % 4 == 1:
+            prm = _with_policy(prm, int(rng.integers(1, 3)), int(rng.integers(1, 3)))
+        r = run.simulate(g, prm)
+        info = {}
+        st, mk, start, fin, cta_sm = stepper.simulate_graph(g, prm, info=info)
+        assert r.status == st
+        if st == 0:
+            assert r.makespan == mk and list(r.start) == start and list(r.finish) == fin
+            assert list(r.busy) == stepper.busy_cycles(g.type, g.work, g.lat_extra, prm, start, mk, info)
+
+
+def test_l2_closed_forms():
+    rng = np.random.default_rng(81)
+    for _ in range(20):
+        k = int(rng.integers(2, 12))
+        w = [int(x) for x in rng.integers(1, 6, k)]
+        # every LOAD a new tile: no hits; one tile reloaded with room for it: all but the first hit
+        distinct = _l2_graph([["LOAD", v, w[v]] for v in range(k)])
+        distinct.n_tiles = k
+        same = _l2_graph([["LOAD", 0, 5] for _ in range(k)])
+        r1 = run.simulate(distinct, _l2_params(1000))
+        r2 = run.simulate(same, _l2_params(5))
+        assert (r1.busy[7], r1.busy[8]) == (0, k)
+        assert (r2.busy[7], r2.busy[8]) == (k - 1, k)
+        # a chain of misses: makespan = sum of (tma_lat + l2_lat + dram_lat + work); hits: 3 + 5 each
+        assert r1.makespan == sum(13 + x for x in w)
+        assert r2.makespan == 18 + (k - 1) * 8
+
+
+def test_l2_parameter_checks():
+    g = _l2_graph([["LOAD", 0, 4]])
+    assert run.simulate(g, _l2_params(8)).status == 0
+    for fields in ((0, 3, 0), (0, 0, 2), (8, -1, 2), (8, 3, 0), (-1, 3, 2)):
+        prm = _l2_params(*fields) if fields[0] >= 0 else _l2_params(8)
+        if fields[0] < 0:
+            prm[W.P_L2_BYTES] = -1
+        assert run.simulate(g, prm).status == run.ERR_INVALID_PARAMS, fields
+    bad = g.subgraph(0)
+    bad.tile = np.array([9], np.uint32)       # tile id >= n_tiles
+    assert run.simulate(bad, _l2_params(8)).status == run.ERR_INVALID_GRAPH
+
+
 def _with_policy(prm, policy, nsub):
     prm = prm.copy()
     prm[W.P_ISSUE_POLICY] = policy
@@ -332,7 +423,7 @@ def test_single_server_no_idle():
         assert r.status == 0
         assert r.makespan == int(g.work.sum())
         assert r.busy[0] == r.makespan          # the tensor server never idles
-        assert list(r.busy[1:]) == [0] * 6
+        assert list(r.busy[1:]) == [0] * 8
 
 
 # ------------------------------------------------------------------ bounds and invariants
