@@ -32,6 +32,8 @@ METRIC = "simulated tile-graph nodes/sec"
 UNIT = "node-points/s"
 KERNEL_SRC = os.path.join(ROOT, "paper_2607_11262_gb300", "csrc", "gts.cu")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_k_simulate.txt")
+ISSUE_FILE = os.path.join(ROOT, "profiles", "issue_k_simulate.txt")
+SCHEDULERS_PER_SM = 4  # warp schedulers per SM; each issues at most one warp-instruction per cycle
 
 
 def node_points_of(graph, params):
@@ -44,12 +46,21 @@ def node_points_of(graph, params):
 
 def algorithmic_bytes(graph, params, full_trace=True):
     """Bytes the batch must move at minimum: the graph read once (node fields
-    1+2+4+4+4+2 B, row pointers, 5 B per edge), 96 B per parameter row, and per
+    1+2+4+4+4+2 B, row pointers, 5 B per edge), the parameter rows, and per
     point its trace (start + finish, 8 B per node), makespan and status."""
     n, m = graph.n_nodes, graph.n_edges
     graph_bytes = n * (1 + 2 + 4 + 4 + 4 + 2) + (n + 1) * 4 + m * 5
     P = int(params.shape[0])
-    return graph_bytes + 96 * P + (8 * node_points_of(graph, params) if full_trace else 0) + 8 * P
+    row = 4 * int(params.shape[1])
+    return graph_bytes + row * P + (8 * node_points_of(graph, params) if full_trace else 0) + 8 * P
+
+
+def profiled(path, name):
+    """A profile figure file, if it was taken on this kernel source and workload."""
+    if not os.path.exists(path):
+        return None
+    f = json.load(open(path))
+    return f if f.get("source_sha256_16") == source_hash() and name in f.get("applies_to", []) else None
 
 
 def source_hash():
@@ -290,10 +301,20 @@ def main():
     peak = float(peaks.get("hbm_gbs", 6800.0))
     achieved = alg / kernel_s / 1e9
     traffic = None
-    if os.path.exists(TRAFFIC_FILE):
-        tf = json.load(open(TRAFFIC_FILE))
-        if tf.get("source_sha256_16") == source_hash() and w.name in tf.get("applies_to", []):
-            traffic = tf["bytes_per_node_point"] * node_points + tf.get("bytes_fixed", 0)
+    tf = profiled(TRAFFIC_FILE, w.name)
+    if tf:
+        traffic = tf["bytes_per_node_point"] * node_points + tf.get("bytes_fixed", 0)
+    # issue-slot roofline: warp-instructions per node (ncu) x node rate against
+    # SMs x schedulers x the SM clock seen during the timed steps
+    issue = None
+    fi = profiled(ISSUE_FILE, w.name)
+    if fi and ck and ck.get("sm_mhz"):
+        sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+        got = fi["warp_instr_per_node_point"] * node_points / kernel_s
+        cap = sms * SCHEDULERS_PER_SM * ck["sm_mhz"] * 1e6
+        issue = {"achieved": got / 1e9, "peak": cap / 1e9, "unit": "Gwarp-instr/s", "frac": got / cap,
+                 "warp_instr_per_node": fi["warp_instr_per_node_point"],
+                 "peak_basis": f"{sms} SMs x {SCHEDULERS_PER_SM} schedulers x {ck['sm_mhz']:.0f} MHz"}
     cb = None
     if not args.no_cpu_baseline:
         cb = cpu_baseline(g, w.params, seconds=args.ref_seconds)
@@ -307,7 +328,7 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": "measured" if peaks else "fallback",
-                     "frac_of_8tbps": achieved / 8000.0},
+                     "frac_of_8tbps": achieved / 8000.0, "issue": issue},
         "cpu_baseline": cb, "e2e": e2e, "gpu_launches": args.steps, "clocks": ck,
         "kernel_source": source_hash(),
     }
