@@ -294,10 +294,11 @@ gts_status gts_params_destroy(gts_params *params);
 uint32_t gts_row_nodes(const gts_graph *graph);
 uint32_t gts_row_ctas(const gts_graph *graph);
 
-/* Device scratch gts_simulate_batch wants: one row of dependency counters per
- * concurrently simulated design point (8 bytes per node of the largest graph,
- * rounded up to 16 bytes).  Returns the size that lets every resident warp
- * work; a smaller scratch (at least one row) runs fewer points at a time.
+/* Device scratch gts_simulate_batch wants: one row per concurrently simulated
+ * design point -- dependency counters (8 bytes per node of the largest graph,
+ * rounded up to 16 bytes) and, for a graph with tiles, one 16-byte L2 list
+ * record per tile.  Returns the size that lets every resident warp work; a
+ * smaller scratch (at least one row) runs fewer points at a time.
  * The kernel clears each row itself; its contents between calls are
  * irrelevant.  Calls sharing one scratch must not overlap on the GPU. */
 size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint32_t flags);
@@ -344,9 +345,10 @@ gts_status gts_results_destroy(gts_results *results);
  *  - The first call on a device looks up that array's address for the current
  *    device (cudaGetSymbolAddress); make that first call before any stream
  *    capture.  No call allocates or frees device memory.
- *  - The graph set's largest graph must have at most GTS_STATIC_SCRATCH_BYTES/8
- *    nodes, else GTS_ERR_NOMEM; fewer design points then run at a time than
- *    with a large caller scratch (one per 8 bytes x nodes of the array).
+ *  - One scratch row (see gts_scratch_bytes) must fit in
+ *    GTS_STATIC_SCRATCH_BYTES, else GTS_ERR_NOMEM: at most 4,194,304 nodes in
+ *    the largest graph without tiles.  Fewer design points then run at a time
+ *    than with a large caller scratch (as many as rows fit in the array).
  *  - All calls share the array and the kernel clears each design point's part
  *    before use, so nothing carries over between calls; calls that overlap on
  *    the GPU (other streams, other threads) race on it and must be ordered by

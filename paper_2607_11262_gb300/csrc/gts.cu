@@ -815,8 +815,6 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       const uint32_t scls = EXT && cls == RC_DSM ? RC_LSU : cls;  // the per-SM class it takes
       busy += (uint32_t)lane == scls ? occ
             : (uint32_t)lane == GTS_BUSY_HBM ? hocc : ((uint32_t)lane == GTS_BUSY_NOC ? nocc : 0u);
-      cn.x = __shfl_sync(FULL, cn.x, 0);
-      cn.y = __shfl_sync(FULL, cn.y, 0);
       // take one free server of the node's class on its SM (lane k tests server k)
       if (cls != RC_NONE) {
         uint32_t *sv = sp + P.L.o_sv + sm * P.L.SC + P.cls_off(scls);
@@ -924,6 +922,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         }
       }
       __syncwarp();
+      cn.x = __shfl_sync(FULL, cn.x, 0);  // the next head's counters (its scratch row is not released into above)
+      cn.y = __shfl_sync(FULL, cn.y, 0);
       set_head(P, i, nx, rn, qn, cn, adj_cnt, adj_rdy);
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
@@ -1593,8 +1593,8 @@ gts_status gts_simulate_batch_noalloc(gts_graph *g, gts_params *P, uint32_t firs
   clear_error();
   if (!g) return fail(GTS_ERR_INVALID_ARG, "null graph");
   if (scratch_row_bytes(g) > GTS_STATIC_SCRATCH_BYTES)
-    return fail(GTS_ERR_NOMEM, "simulate_noalloc: a graph of the set has more nodes than the static scratch holds "
-                               "(GTS_STATIC_SCRATCH_BYTES / 8)");
+    return fail(GTS_ERR_NOMEM, "simulate_noalloc: one scratch row (8 bytes per node of the largest graph, 16 per "
+                               "tile) does not fit in the static scratch (GTS_STATIC_SCRATCH_BYTES)");
   void *scr = nullptr;
   gts_status st = static_scratch(&scr);
   if (st != GTS_OK) return st;
