@@ -17,7 +17,11 @@ the speedup and the NoC utilisation (busy NoC cycles / (servers x makespan)).
 The L2 study runs the persistent GEMM of ``l2gemm`` in row-major and grouped
 rasterization at L2 capacities of 0-100 MB and reports makespan and hit rate.
 
-    python -m paper_2607_11262_gb300.study [--study pipelines|noc|l2] [--points-per-graph 64] [--json out.json]
+The policy study reruns workloads' design points under the per-subpartition
+issue policies (greedy-then-oldest, round-robin; Section 5.3) with 1, 2 and 4
+schedulers per SM and compares each makespan with the lowest-id order.
+
+    python -m paper_2607_11262_gb300.study [--study pipelines|noc|l2|policies] [--points-per-graph 64] [--json out.json]
 """
 from __future__ import annotations
 
@@ -26,7 +30,7 @@ import json
 
 import numpy as np
 
-from . import clusters, gts, l2gemm, pipelines
+from . import clusters, gts, l2gemm, pipelines, workloads
 
 
 def run_study(points_per_graph=1, device="cuda"):
@@ -122,6 +126,53 @@ def run_l2_study(device="cuda"):
     return rows
 
 
+POLICY_CASES = (("gto", 1), ("gto", 2), ("gto", 4), ("rr", 1), ("rr", 2), ("rr", 4))
+
+
+def run_policy_study(names=("gemm512", "wsgemm_small", "fa_fwd"), points=64, device="cuda"):
+    """Makespan under each issue policy relative to lowest-id, per workload:
+    one dict per (workload, policy, schedulers) with the ratio's min / mean /
+    max over the points."""
+    import torch
+    gts.load()
+    code = {"gto": workloads.POLICY_GTO, "rr": workloads.POLICY_RR}
+    rows = []
+    for name in names:
+        w = workloads.workload(name)
+        idx = np.linspace(0, w.params.shape[0] - 1, min(points, w.params.shape[0])).round().astype(int)
+        base = w.params[idx]
+        variants = [base]
+        for pol, nsub in POLICY_CASES:
+            p = base.copy()
+            p[:, workloads.P_ISSUE_POLICY] = code[pol]
+            p[:, workloads.P_SUBPARTITIONS] = nsub
+            variants.append(p)
+        table = np.ascontiguousarray(np.concatenate(variants), np.int32)
+        dg = gts.DeviceGraph(w.graph, device=device)
+        dp = gts.DeviceParams(dg, table)
+        out = gts.simulate(dg, dp, flags=0)
+        torch.cuda.synchronize()
+        status = out.status.cpu().numpy()
+        if np.any(status != gts.GTS_OK):
+            raise gts.GtsError(int(status[status != 0][0]), "a study point did not simulate")
+        mk = out.makespan.cpu().numpy().reshape(len(variants), len(idx)).astype(np.float64)
+        dp.close()
+        dg.close()
+        for k, (pol, nsub) in enumerate(POLICY_CASES):
+            r = mk[k + 1] / mk[0]
+            rows.append(dict(workload=name, policy=pol, schedulers=nsub, points=len(idx), ratio_min=float(r.min()),
+                             ratio_mean=float(r.mean()), ratio_max=float(r.max())))
+    return rows
+
+
+def format_policy_table(rows):
+    lines = [f"{'workload':<14}{'policy':<8}{'schedulers':>11}{'makespan / lowest-id (min / mean / max)':>42}"]
+    for r in rows:
+        lines.append(f"{r['workload']:<14}{r['policy']:<8}{r['schedulers']:>11}"
+                     f"{r['ratio_min']:>24.3f} / {r['ratio_mean']:.3f} / {r['ratio_max']:.3f}")
+    return "\n".join(lines)
+
+
 def format_l2_table(rows):
     lines = [f"{'order':<10}{'L2 MB':>7}{'cycles':>12}{'hits':>9}{'loads':>9}{'hit rate':>10}"]
     for r in rows:
@@ -153,7 +204,7 @@ def format_table(rows):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--study", default="pipelines", choices=["pipelines", "noc", "l2"])
+    ap.add_argument("--study", default="pipelines", choices=["pipelines", "noc", "l2", "policies"])
     ap.add_argument("--points-per-graph", type=int, default=1)
     ap.add_argument("--json", default=None)
     args = ap.parse_args()
@@ -163,6 +214,9 @@ def main():
     elif args.study == "l2":
         rows = run_l2_study()
         print(format_l2_table(rows))
+    elif args.study == "policies":
+        rows = run_policy_study(points=args.points_per_graph)
+        print(format_policy_table(rows))
     else:
         rows = run_study(args.points_per_graph)
         print(format_table(rows))

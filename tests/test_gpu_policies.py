@@ -120,3 +120,20 @@ def test_policy_rows_validated_per_point():
     assert res["status"][0] == 0
     assert list(res["status"][1:]) == [-3, -3, -3, -3]
     _check_all(g, p, res)
+
+
+def test_policy_study_matches_oracle():
+    from paper_2607_11262_gb300 import study
+    rows = study.run_policy_study(names=("gemm512",), points=3)
+    w = W.workload("gemm512")
+    idx = np.linspace(0, w.params.shape[0] - 1, 3).round().astype(int)
+    base = [oracle_run.simulate(w.graph, w.params[q]).makespan for q in idx]
+    code = {"gto": W.POLICY_GTO, "rr": W.POLICY_RR}
+    for r in rows:
+        ratios = []
+        for q, b in zip(idx, base):
+            p = w.params[q].copy()
+            p[W.P_ISSUE_POLICY], p[W.P_SUBPARTITIONS] = code[r["policy"]], r["schedulers"]
+            ratios.append(oracle_run.simulate(w.graph, p).makespan / b)
+        assert r["ratio_min"] == pytest.approx(min(ratios), rel=1e-12)
+        assert r["ratio_max"] == pytest.approx(max(ratios), rel=1e-12)
