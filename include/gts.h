@@ -289,18 +289,32 @@ gts_status gts_params_upload(gts_graph *graph, const int32_t *d_params, uint32_t
                              void *stream, gts_params **out);
 gts_status gts_params_destroy(gts_params *params);
 
+/* Attaches a processing order to a parameter table.  Fills d_order (device,
+ * [n_points] uint32, caller-owned, borrowed by params) with the point indices
+ * sorted by estimated cost, largest first (nodes of the row's graph x (743 +
+ * simulated SMs), x 3.5 for rows that need the extended model), and makes
+ * gts_simulate_batch hand points to its warps in that order, each warp taking
+ * the next point when it finishes one (longest processing time first, which
+ * keeps the last wave short).  Results do not depend on the order.  Without
+ * one, warp w takes points w, w + warps, ... .  Waits for `stream`.
+ * Errors: INVALID_ARG, CUDA. */
+gts_status gts_params_set_order(gts_params *params, uint32_t *d_order, void *stream);
+
 /* Per-point output row lengths: start/finish rows hold gts_row_nodes() entries
  * (the largest graph of the stack), cta_sm rows gts_row_ctas(). */
 uint32_t gts_row_nodes(const gts_graph *graph);
 uint32_t gts_row_ctas(const gts_graph *graph);
 
-/* Device scratch gts_simulate_batch wants: one row per concurrently simulated
- * design point -- dependency counters (8 bytes per node of the largest graph,
- * rounded up to 16 bytes) and, for a graph with tiles, one 16-byte L2 list
- * record per tile.  Returns the size that lets every resident warp work; a
- * smaller scratch (at least one row) runs fewer points at a time.
+/* Device scratch gts_simulate_batch wants: GTS_SCRATCH_HEADER_BYTES (the
+ * next-point counter of an ordered batch), then one row per concurrently
+ * simulated design point -- dependency counters (8 bytes per node of the
+ * largest graph, rounded up to 16 bytes) and, for a graph with tiles, one
+ * 16-byte L2 list record per tile.  Returns the size that lets every resident
+ * warp work; a smaller scratch (the header and at least one row) runs fewer
+ * points at a time.
  * The kernel clears each row itself; its contents between calls are
  * irrelevant.  Calls sharing one scratch must not overlap on the GPU. */
+#define GTS_SCRATCH_HEADER_BYTES 16
 size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint32_t flags);
 
 /*
@@ -345,8 +359,8 @@ gts_status gts_results_destroy(gts_results *results);
  *  - The first call on a device looks up that array's address for the current
  *    device (cudaGetSymbolAddress); make that first call before any stream
  *    capture.  No call allocates or frees device memory.
- *  - One scratch row (see gts_scratch_bytes) must fit in
- *    GTS_STATIC_SCRATCH_BYTES, else GTS_ERR_NOMEM: at most 4,194,304 nodes in
+ *  - The scratch header and one row (see gts_scratch_bytes) must fit in
+ *    GTS_STATIC_SCRATCH_BYTES, else GTS_ERR_NOMEM: about 4.19 million nodes in
  *    the largest graph without tiles.  Fewer design points then run at a time
  *    than with a large caller scratch (as many as rows fit in the array).
  *  - All calls share the array and the kernel clears each design point's part

@@ -612,6 +612,28 @@ __device__ __forceinline__ uint32_t l2_access(uint4 *T, uint32_t x, uint32_t b, 
   return e.w;
 }
 
+// The next design point of a warp (batch-relative), or NONE: from the shared
+// counter over `order` (skipping points outside the batch), else the warp's
+// own stride.
+__device__ __noinline__ uint32_t next_point_of(const uint32_t *order, uint32_t n_order, uint32_t *counter,
+                                               uint32_t first, uint32_t n, uint32_t q, uint32_t stride, int lane) {
+  if (!order) return q + stride < n ? q + stride : NONE;
+  for (;;) {
+    uint32_t k = 0;
+    if (lane == 0) k = atomicAdd(counter, 1u);
+    k = __shfl_sync(FULL, k, 0);
+    if (k >= n_order) return NONE;
+    const uint32_t pa = order[k];
+    if (pa >= first && pa - first < n) return pa - first;
+  }
+}
+
+__device__ __forceinline__ uint32_t first_point_of(const uint32_t *order, uint32_t n_order, uint32_t *counter,
+                                                   uint32_t first, uint32_t n, uint32_t gw, int lane) {
+  if (!order) return gw < n ? gw : NONE;
+  return next_point_of(order, n_order, counter, first, n, 0u, 0u, lane);
+}
+
 // EXT: the kernel instance that also runs the per-subpartition issue policies
 // and the NoC of DSMEM nodes; the host launches the plain instance when no row
 // asks for a policy and the graph has no DSMEM node.
@@ -619,7 +641,8 @@ template <bool EXT>
 __global__ void __launch_bounds__(MAX_WPB * 32, 1)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
-           int32_t *d_cta_sm, int64_t *d_busy, uint2 *scratch, uint32_t n_warps, uint32_t budget_words) {
+           int32_t *d_cta_sm, int64_t *d_busy, uint2 *scratch, uint32_t n_warps, uint32_t budget_words,
+           const uint32_t *__restrict__ order, uint32_t n_order) {
   extern __shared__ __align__(16) uint32_t smem[];
   const int lane = threadIdx.x & 31;
   const uint32_t wib = threadIdx.x >> 5;
@@ -631,7 +654,11 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
   uint32_t *sp = P.sp;
   const bool want_digest = d_digest != nullptr;
 
-  for (uint32_t q = gw; q < n_points; q += n_warps) {
+  // points: the next one in `order` (a counter in the scratch header), or
+  // gw, gw + n_warps, ... without an order
+  uint32_t *next_point = reinterpret_cast<uint32_t *>(scratch);
+  for (uint32_t q = first_point_of(order, n_order, next_point, first_point, n_points, gw, lane); q != NONE;
+       q = next_point_of(order, n_order, next_point, first_point, n_points, q, n_warps, lane)) {
     const uint32_t p = first_point + q;
     // ---- parameter row -> shared memory
     if (lane < GTS_NPARAM) sp[lane] = (uint32_t)params[(size_t)p * GTS_NPARAM + lane];
@@ -664,7 +691,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     P.policy = (uint32_t)prm[GTS_P_ISSUE_POLICY];
     P.st = (flags & GTS_FULL_TRACE) ? d_start + (size_t)q * g.row_nodes : nullptr;
     P.fi = (flags & GTS_FULL_TRACE) ? d_finish + (size_t)q * g.row_nodes : nullptr;
-    P.scr = scratch + (size_t)gw * (((g.row_nodes + 1u) & ~1u) + 2u * g.n_tiles);
+    P.scr = scratch + GTS_SCRATCH_HEADER_BYTES / 8 + (size_t)gw * (((g.row_nodes + 1u) & ~1u) + 2u * g.n_tiles);
     uint4 *l2t = reinterpret_cast<uint4 *>(P.scr + ((g.row_nodes + 1u) & ~1u));  // L2 list records per tile
     int32_t *cta_sm_row = (flags & GTS_WANT_CTA_SM) ? d_cta_sm + (size_t)q * g.row_ctas : nullptr;
 
@@ -1018,6 +1045,8 @@ struct gts_params {
   uint32_t n_points;
   std::vector<uint32_t> words;  // per row: shared words, 0 if the row is invalid or too large
   std::vector<uint8_t> sched;   // per row: asks for a per-subpartition issue policy or the L2 model
+  std::vector<double> cost;     // per row: estimated simulation cost (0 for invalid rows)
+  const uint32_t *d_order = nullptr;  // processing order (gts_params_set_order), borrowed
 };
 
 struct gts_results {
@@ -1394,15 +1423,35 @@ gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_p
   P->n_points = n_points;
   P->words.assign(n_points, 0u);
   P->sched.assign(n_points, 0u);
+  P->cost.assign(n_points, 0.0);
   for (uint32_t p = 0; p < n_points; p++) {
     const int32_t *row = h.data() + (size_t)p * GTS_NPARAM;
     if (check_row(row, g->G, g->dg.class_mask) != GTS_OK) continue;
     P->sched[p] = row[GTS_P_ISSUE_POLICY] != GTS_POLICY_LOWEST_ID || row[GTS_P_L2_BYTES] != 0;
     const uint32_t gi = (uint32_t)row[GTS_P_GRAPH_INDEX];
     Layout L;
-    if (make_layout(row, g->cta_off[gi + 1] - g->cta_off[gi], g->W, g->dg.class_mask, L)) P->words[p] = L.words;
+    if (make_layout(row, g->cta_off[gi + 1] - g->cta_off[gi], g->W, g->dg.class_mask, L)) {
+      P->words[p] = L.words;
+      // per issue the work grows slowly with the simulated SMs; the extended model costs about 3.5x
+      P->cost[p] = (double)(g->node_off[gi + 1] - g->node_off[gi]) * (743.0 + L.NS) * (P->sched[p] ? 3.5 : 1.0);
+    }
   }
   *out = P;
+  return GTS_OK;
+}
+
+gts_status gts_params_set_order(gts_params *P, uint32_t *d_order, void *stream) {
+  clear_error();
+  if (!P || (P->n_points && !d_order)) return fail(GTS_ERR_INVALID_ARG, "null params or order");
+  std::vector<uint32_t> order(P->n_points);
+  for (uint32_t p = 0; p < P->n_points; p++) order[p] = p;
+  std::stable_sort(order.begin(), order.end(), [&](uint32_t a, uint32_t b) { return P->cost[a] > P->cost[b]; });
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaSuccess;
+  if (P->n_points) e = cudaMemcpyAsync(d_order, order.data(), (size_t)P->n_points * 4, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "params_set_order: copy to device");
+  P->d_order = d_order;
   return GTS_OK;
 }
 
@@ -1415,8 +1464,9 @@ namespace {
 // Per-warp scratch: one (released-predecessor count, max release cycle) pair
 // per node of the largest graph, rounded to 16 bytes.
 // ... plus, for a graph with tiles, one 16-byte L2 list record per tile.
+// At least 16 bytes, so that a graph without nodes still has a row size to divide by.
 uint64_t scratch_row_bytes(const gts_graph *g) {
-  return (((uint64_t)g->dg.row_nodes + 1) & ~1ull) * 8 + 16ull * g->dg.n_tiles;
+  return std::max<uint64_t>(16, (((uint64_t)g->dg.row_nodes + 1) & ~1ull) * 8 + 16ull * g->dg.n_tiles);
 }
 
 struct Plan {
@@ -1461,7 +1511,7 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
   warps = std::min<uint64_t>(warps, np);
   if (limit_by_scratch) {
     const uint64_t row = scratch_row_bytes(g);
-    const uint64_t fit = scratch_bytes / row;
+    const uint64_t fit = scratch_bytes > GTS_SCRATCH_HEADER_BYTES ? (scratch_bytes - GTS_SCRATCH_HEADER_BYTES) / row : 0;
     if (fit == 0) return fail(GTS_ERR_NOMEM, "scratch smaller than one design point's counter row");
     warps = std::min(warps, fit);
   }
@@ -1477,7 +1527,7 @@ size_t gts_scratch_bytes(const gts_graph *g, const gts_params *P, uint32_t flags
   if (!g || !P) return 0;
   Plan pl;
   if (plan_launch(g, P, 0, P->n_points, flags, 0, false, pl) != GTS_OK) return 0;
-  return (size_t)pl.warps * scratch_row_bytes(g);
+  return GTS_SCRATCH_HEADER_BYTES + (size_t)pl.warps * scratch_row_bytes(g);
 }
 
 gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point, uint32_t n_points, uint32_t flags,
@@ -1504,11 +1554,16 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
     Plan pl;
     gts_status st = plan_launch(g, P, first_point, n_points, flags, scratch_bytes, true, pl);
     if (st != GTS_OK) return st;
+    if (P->d_order) {  // the next-point counter
+      const cudaError_t em = cudaMemsetAsync(d_scratch, 0, GTS_SCRATCH_HEADER_BYTES, s);
+      if (em != cudaSuccess) return cuda_fail(em, "simulate: clear the point counter");
+    }
     auto kern = pl.sched ? k_simulate<true> : k_simulate<false>;
     kern<<<pl.blocks, pl.wpb * 32, pl.smem, s>>>(
         g->dg, P->d_params, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status,
         (flags & GTS_WANT_DIGEST) ? d_digest : nullptr, (flags & GTS_WANT_CTA_SM) ? d_cta_sm : nullptr,
-        (flags & GTS_WANT_BUSY) ? d_busy : nullptr, (uint2 *)d_scratch, pl.warps, pl.words);
+        (flags & GTS_WANT_BUSY) ? d_busy : nullptr, (uint2 *)d_scratch, pl.warps, pl.words, P->d_order,
+        P->d_order ? P->n_points : 0u);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "simulate: launch");
   }
@@ -1592,7 +1647,7 @@ gts_status gts_simulate_batch_noalloc(gts_graph *g, gts_params *P, uint32_t firs
                                       void *stream) {
   clear_error();
   if (!g) return fail(GTS_ERR_INVALID_ARG, "null graph");
-  if (scratch_row_bytes(g) > GTS_STATIC_SCRATCH_BYTES)
+  if (GTS_SCRATCH_HEADER_BYTES + scratch_row_bytes(g) > GTS_STATIC_SCRATCH_BYTES)
     return fail(GTS_ERR_NOMEM, "simulate_noalloc: one scratch row (8 bytes per node of the largest graph, 16 per "
                                "tile) does not fit in the static scratch (GTS_STATIC_SCRATCH_BYTES)");
   void *scr = nullptr;

@@ -43,9 +43,10 @@ GTS_NPARAM = 32
 GTS_POLICY_LOWEST_ID, GTS_POLICY_GTO, GTS_POLICY_RR = 0, 1, 2
 
 GTS_STATIC_SCRATCH_BYTES = 32 << 20
+GTS_SCRATCH_HEADER_BYTES = 16
 
 EXPORTS = ("gts_graph_workspace_bytes", "gts_graph_create", "gts_graph_destroy", "gts_template_workspace_bytes",
-           "gts_graph_create_templated", "gts_params_upload",
+           "gts_graph_create_templated", "gts_params_upload", "gts_params_set_order",
            "gts_params_destroy", "gts_row_nodes", "gts_row_ctas", "gts_scratch_bytes", "gts_simulate_batch",
            "gts_read_results", "gts_results_destroy", "gts_simulate_batch_noalloc", "gts_last_error")
 
@@ -105,6 +106,8 @@ def load():
     lib.gts_params_upload.restype = i32
     lib.gts_params_destroy.argtypes = [vp]
     lib.gts_params_destroy.restype = i32
+    lib.gts_params_set_order.argtypes = [vp, vp, vp]
+    lib.gts_params_set_order.restype = i32
     lib.gts_row_nodes.argtypes = [vp]
     lib.gts_row_nodes.restype = u32
     lib.gts_row_ctas.argtypes = [vp]
@@ -164,6 +167,10 @@ def gts_params_upload(graph, d_params: int, n_points: int, stream: int = 0):
 
 def gts_params_destroy(params):
     _check(load().gts_params_destroy(params))
+
+
+def gts_params_set_order(params, d_order: int, stream: int = 0):
+    _check(load().gts_params_set_order(params, d_order, stream))
 
 
 def gts_row_nodes(graph):
@@ -326,7 +333,9 @@ class DeviceGraph:
 class DeviceParams:
     """A [P][GTS_NPARAM] int32 parameter table resident on the GPU."""
 
-    def __init__(self, dgraph: DeviceGraph, params, stream=None, tensor=None, n_points=None):
+    def __init__(self, dgraph: DeviceGraph, params, stream=None, tensor=None, n_points=None, ordered=True):
+        """``ordered``: hand points to the warps largest estimated cost first
+        (gts_params_set_order); results are the same either way."""
         import torch
         self.dgraph = dgraph
         if tensor is None:
@@ -339,10 +348,14 @@ class DeviceParams:
             self.n_points = int(n_points)
             self.tensor = tensor
         self.handle = gts_params_upload(dgraph.handle, self.tensor.data_ptr(), self.n_points, _stream_handle(stream))
+        self.order = None
+        if ordered and self.n_points:
+            self.order = torch.empty(self.n_points, dtype=torch.int32, device=self.tensor.device)
+            gts_params_set_order(self.handle, self.order.data_ptr(), _stream_handle(stream))
 
     @classmethod
-    def from_device_tensor(cls, dgraph, tensor, n_points, stream=None):
-        return cls(dgraph, None, stream=stream, tensor=tensor, n_points=n_points)
+    def from_device_tensor(cls, dgraph, tensor, n_points, stream=None, ordered=True):
+        return cls(dgraph, None, stream=stream, tensor=tensor, n_points=n_points, ordered=ordered)
 
     def close(self):
         if getattr(self, "handle", None):

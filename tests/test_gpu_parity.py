@@ -143,14 +143,15 @@ def test_makespan_only_with_tiny_scratch():
     dg = gts.DeviceGraph(w.graph)
     dp = gts.DeviceParams(dg, w.params)
     row = ((dg.row_nodes + 1) // 2 * 2) * 8
-    scratch = torch.empty(3 * row, dtype=torch.uint8, device="cuda")  # 3 design points at a time
+    head = gts.GTS_SCRATCH_HEADER_BYTES
+    scratch = torch.empty(head + 3 * row, dtype=torch.uint8, device="cuda")  # 3 design points at a time
     out = gts.simulate(dg, dp, flags=gts.GTS_WANT_DIGEST, scratch=scratch)
     torch.cuda.synchronize()
     full = H.run_gpu(w.graph, w.params)
     assert np.array_equal(out.makespan.cpu().numpy(), full["makespan"])
     assert np.array_equal(out.digest.cpu().numpy().astype(np.uint64), full["digest"])
     with pytest.raises(gts.GtsError) as e:
-        small = torch.empty(row - 8, dtype=torch.uint8, device="cuda")
+        small = torch.empty(head + row - 16, dtype=torch.uint8, device="cuda")
         gts.simulate(dg, dp, flags=0, scratch=small)
     assert e.value.status == gts.GTS_ERR_NOMEM
 
