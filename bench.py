@@ -358,7 +358,8 @@ def measure_e2e(graph, params, gts, stream, reps=2, templates=None):
     hp = torch.from_numpy(np.ascontiguousarray(params, np.int32).reshape(-1)).pin_memory()
     h_mk = torch.empty(P, dtype=torch.int32).pin_memory()
     h_st = torch.empty(P, dtype=torch.int32).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for t in host.values()) + hp.numel() * 4
+    # inputs, plus the processing order libgts uploads (4 B per point, gts_params_set_order)
+    h2d = sum(t.numel() * t.element_size() for t in host.values()) + hp.numel() * 4 + 4 * P
     d2h = P * 8
     flags = gts.GTS_FULL_TRACE
     times = []
