@@ -636,9 +636,12 @@ __device__ __forceinline__ uint32_t first_point_of(const uint32_t *order, uint32
 
 // EXT: the kernel instance that also runs the per-subpartition issue policies
 // and the NoC of DSMEM nodes; the host launches the plain instance when no row
-// asks for a policy and the graph has no DSMEM node.
+// asks for a policy and the graph has no DSMEM node.  The plain instance is
+// held to 128 registers: a warp's registers come from one SM sub-partition's
+// 16K-register file, so at 129-170 registers only 3 warps fit per
+// sub-partition (12 per SM) instead of the 14 shared memory allows.
 template <bool EXT>
-__global__ void __launch_bounds__(MAX_WPB * 32, 1)
+__global__ void __launch_bounds__(MAX_WPB * 32, EXT ? 1 : 4)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
            int32_t *d_cta_sm, int64_t *d_busy, uint2 *scratch, uint32_t n_warps, uint32_t budget_words,
