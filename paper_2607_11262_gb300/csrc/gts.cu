@@ -244,6 +244,12 @@ __device__ __forceinline__ uint32_t cdiv_c(uint32_t n, uint32_t d, uint64_t M) {
   return q + (q * d != n ? 1u : 0u);
 }
 
+// floor(n / d) for n < 2^16 from m = div16_const(d) = ceil(2^32 / d) (0 for d = 1):
+// n*m/2^32 exceeds n/d by less than n/2^32 < 2^-16, never enough to carry past the
+// next integer when d < 2^16; for larger d both sides are 0.
+__host__ __device__ __forceinline__ uint32_t div16_const(uint32_t d) { return d <= 1u ? 0u : 0xFFFFFFFFu / d + 1u; }
+__device__ __forceinline__ uint32_t div16(uint32_t n, uint32_t m) { return m ? __umulhi(n, m) : n; }
+
 __device__ __forceinline__ uint64_t mix64(uint64_t z) {  // splitmix64 finaliser (Steele, Lea, Flood 2014)
   z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
   z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
@@ -276,6 +282,9 @@ struct Pt {
   uint64_t offs;     // byte r: offset of class r's servers inside an SM's servers
   uint32_t caps;     // 6 bits per class: servers of class r (0: class unused)
   uint32_t policy;   // GTS_POLICY_*; L.nsub > 0 for the per-subpartition policies
+  uint32_t mW, mCps; // div16 constants of W and ctas_per_sm; slot and CTA-slot indices stay below
+                     // 2^16 because 5-word slot records of a point fit in MAX_SMEM_BYTES
+  uint32_t mSub, mCsms;  // div16 constants of the scheduler count and the SMs per NoC group
   __device__ __forceinline__ uint32_t cls_off(uint32_t r) const { return (uint32_t)(offs >> (8 * r)) & 255u; }
   __device__ __forceinline__ uint32_t cls_cap(uint32_t r) const { return (caps >> (6 * r)) & 63u; }
   __device__ __forceinline__ uint32_t *slot(uint32_t i) const { return sp + L.o_slot + i * SLOT_WORDS; }
@@ -310,7 +319,7 @@ __device__ __forceinline__ void node_cost(const uint32_t *sp, uint32_t type, uin
 
 // Key of slot i computed at cycle t (>= t; INF if it cannot issue yet).
 template <bool EXT>
-__device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t) {
+__device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t sm, uint32_t t) {
   const uint32_t *sl = P.slot(i);
   const uint32_t h = sl[F_HID];
   const uint32_t meta = sl[F_META];
@@ -318,7 +327,6 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
   uint32_t k = max(sl[F_RDY], t);
   const uint32_t cls = meta & 7u;
   if (cls != RC_NONE) {
-    const uint32_t sm = i / P.L.per;
     const uint32_t sc = EXT && cls == RC_DSM ? RC_LSU : cls;
     const uint32_t *sv = P.sp + P.L.o_sv + sm * P.L.SC + P.cls_off(sc);
     const uint32_t cap = P.cls_cap(sc);
@@ -326,7 +334,7 @@ __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t t
     for (uint32_t q = 1; q < cap; q++) a = min(a, sv[q]);
     k = max(k, a);
     if (EXT && cls == RC_DSM) {  // and a NoC server of the SM's group
-      const uint32_t *ns = P.sp + P.L.o_ns + (sm / P.L.csms) * P.L.cap_noc;
+      const uint32_t *ns = P.sp + P.L.o_ns + div16(sm, P.mCsms) * P.L.cap_noc;
       a = ns[0];
       for (uint32_t q = 1; q < P.L.cap_noc; q++) a = min(a, ns[q]);
       k = max(k, a);
@@ -350,7 +358,7 @@ __device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t 
     const uint32_t *sq = P.sub(s, u);
     uint32_t m = INF;
     for (uint32_t l = u; l < nl; l += nsub) {
-      const uint32_t k = slot_key<EXT>(P, i0 + l, t);
+      const uint32_t k = slot_key<EXT>(P, i0 + l, s, t);
       if (k == INF) continue;
       if (P.slot(i0 + l)[F_HID] & HBM_BIT) {
         hmin = min(hmin, k);
@@ -363,15 +371,17 @@ __device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t 
     const uint32_t E = max(m, sq[Q_AVAIL]), last = sq[Q_LAST];
     uint64_t bp = INF64;  // (policy key << 32 | slot)
     for (uint32_t l = u; l < nl; l += nsub) {
-      const uint32_t k = slot_key<EXT>(P, i0 + l, t);
+      const uint32_t k = slot_key<EXT>(P, i0 + l, s, t);
       if (k == INF) continue;
       const uint32_t e = (P.slot(i0 + l)[F_HID] & HBM_BIT) ? max(k, H) : k;
       if (e > E) continue;
       uint32_t key;
       if (P.policy == GTS_POLICY_GTO) {  // greedy slot, then the oldest warp (CTA id, warp)
-        key = (l == last ? 0u : 0x80000000u) | (P.cta((i0 + l) / P.W)[C_ID] * P.W + l % P.W);
+        const uint32_t cs = div16(i0 + l, P.mW);  // CTA slot; i0 is a multiple of W
+        key = (l == last ? 0u : 0x80000000u) | (P.cta(cs)[C_ID] * P.W + (i0 + l - cs * P.W));
       } else {                            // round-robin after the last slot
-        key = last == NONE ? l : (l + per - last - 1u) % per;
+        const uint32_t x = l + per - last - 1u;  // l, last < per
+        key = last == NONE ? l : (x >= per ? x - per : x);
       }
       bp = min(bp, pack(key, l));
     }
@@ -405,7 +415,7 @@ __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, 
     const uint32_t i = base + lane;
     uint64_t val = INF64;
     if (i < i1) {
-      const uint32_t k = slot_key<EXT>(P, i, t);
+      const uint32_t k = slot_key<EXT>(P, i, s, t);
       const uint32_t h = P.slot(i)[F_HID];
       if (k != INF) {
         const bool hb = (h & HBM_BIT) != 0u;
@@ -442,7 +452,7 @@ __device__ __forceinline__ void rescan_sm_lane(const Pt &P, uint32_t s, uint32_t
   uint64_t best = INF64;
   uint32_t bsl = 0, hmin = INF;
   for (uint32_t i = i0; i < i1; i++) {
-    const uint32_t k = slot_key<EXT>(P, i, t);
+    const uint32_t k = slot_key<EXT>(P, i, s, t);
     if (k == INF) continue;
     const uint32_t h = P.slot(i)[F_HID];
     const bool hb = (h & HBM_BIT) != 0u;
@@ -558,7 +568,7 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
       cr[C_ID] = c;
       cr[C_REM] = cnt;
       cr[C_END] = 0u;
-      if (cta_sm_row) cta_sm_row[c - P.c0] = (int32_t)(freeslot / P.cps);
+      if (cta_sm_row) cta_sm_row[c - P.c0] = (int32_t)div16(freeslot, P.mCps);
       __threadfence();  // lane 0's earlier counter releases before the heads are read below
     }
     __syncwarp();
@@ -576,7 +586,7 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
       set_head(P, i, v, r, q, cc, 0u, 0u);
     }
     __syncwarp();
-    const uint32_t s = freeslot / P.cps;
+    const uint32_t s = div16(freeslot, P.mCps);
     refresh_sm<EXT>(P, s, t, C.H, lane);
     refresh_owner(P, s & 31u, lane, b, bsl);
     C.next_cta++;
@@ -636,12 +646,13 @@ __device__ __forceinline__ uint32_t first_point_of(const uint32_t *order, uint32
 
 // EXT: the kernel instance that also runs the per-subpartition issue policies
 // and the NoC of DSMEM nodes; the host launches the plain instance when no row
-// asks for a policy and the graph has no DSMEM node.  The plain instance is
-// held to 128 registers: a warp's registers come from one SM sub-partition's
-// 16K-register file, so at 129-170 registers only 3 warps fit per
-// sub-partition (12 per SM) instead of the 14 shared memory allows.
+// asks for a policy and the graph has no DSMEM node.  A warp's registers come
+// from one SM sub-partition's 16K-register file, allocated 8 per thread at a
+// time: 4 warps fit per sub-partition up to 128 registers, 3 up to 168, 2
+// above.  The plain instance is held to 128 (16 warps per SM; shared memory
+// allows 14 on the large rows), the extended one to 168 (12 warps per SM).
 template <bool EXT>
-__global__ void __launch_bounds__(MAX_WPB * 32, EXT ? 1 : 4)
+__global__ void __launch_bounds__(MAX_WPB * 32, EXT ? 3 : 4)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
            int32_t *d_cta_sm, int64_t *d_busy, uint2 *scratch, uint32_t n_warps, uint32_t budget_words,
@@ -691,6 +702,10 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       continue;
     }
     P.cps = (uint32_t)prm[GTS_P_CTAS_PER_SM];
+    P.mW = div16_const(P.W);
+    P.mCps = div16_const(P.cps);
+    P.mSub = EXT ? div16_const(P.L.nsub) : 0u;
+    P.mCsms = EXT ? div16_const(P.L.csms) : 0u;
     P.policy = (uint32_t)prm[GTS_P_ISSUE_POLICY];
     P.st = (flags & GTS_FULL_TRACE) ? d_start + (size_t)q * g.row_nodes : nullptr;
     P.fi = (flags & GTS_FULL_TRACE) ? d_finish + (size_t)q * g.row_nodes : nullptr;
@@ -804,8 +819,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       const uint32_t v = (uint32_t)m;
       const uint32_t i = __shfl_sync(FULL, bsl, owner);
       const uint32_t t = C.t;
-      const uint32_t cs = i / P.W;
-      const uint32_t sm = cs / P.cps;
+      const uint32_t cs = div16(i, P.mW);
+      const uint32_t sm = div16(cs, P.mCps);
       const uint32_t *sl = P.slot(i);
       const uint32_t hidv = sl[F_HID], meta = sl[F_META], nx = sl[F_NXT], sb = sl[F_SB];
       const uint32_t cls = meta & 7u;
@@ -854,7 +869,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       }
       bool noc_touch = false;  // a NoC server of the SM's group was taken
       if (EXT && cls == RC_DSM) {
-        uint32_t *ns = sp + P.L.o_ns + (sm / P.L.csms) * P.L.cap_noc;
+        uint32_t *ns = sp + P.L.o_ns + div16(sm, P.mCsms) * P.L.cap_noc;
         const bool fr = (uint32_t)lane < P.L.cap_noc && ns[lane] <= t;
         const uint32_t bal = __ballot_sync(FULL, fr);
         if (lane == __ffs(bal) - 1) ns[lane] = t + nocc;
@@ -862,7 +877,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       }
       if (EXT && P.L.nsub && lane == 0) {  // the issuing scheduler: one issue per cycle, remember the slot
         const uint32_t l = i - sm * P.L.per;
-        uint32_t *sq = P.sub(sm, l % P.L.nsub);
+        uint32_t *sq = P.sub(sm, l - div16(l, P.mSub) * P.L.nsub);
         sq[Q_AVAIL] = t + 1u;
         sq[Q_LAST] = l;
       }
@@ -977,7 +992,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
           refresh_owner(P, sm & 31u, lane, b, bsl);
         }
         if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
-          const uint32_t g0 = (sm / P.L.csms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
+          const uint32_t g0 = div16(sm, P.mCsms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
           for (uint32_t s = g0 + lane; s < g1; s += 32)
             if (s != sm) rescan_sm_lane<EXT>(P, s, t, C.H);
           __syncwarp();
