@@ -399,12 +399,69 @@ __device__ __forceinline__ void rescan_sm_sub(const Pt &P, uint32_t s, uint32_t 
   o[3] = hmin;
 }
 
+// Warp-parallel form of rescan_sm_sub for SMs of at most 32 slots (one slot
+// per lane): each lane keys its slot once; per scheduler one reduction gives
+// E_u and a second its pick (policy keys are distinct within a scheduler).
+template <bool EXT>
+__device__ __forceinline__ void rescan_sm_sub_warp(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane) {
+  const uint32_t per = P.L.per, nsub = P.L.nsub, i0 = s * per;
+  const uint32_t nl = min(per, P.L.S - i0);
+  const uint32_t l = (uint32_t)lane;
+  uint32_t e = INF, hk = INF, id = 0, u = NONE;
+  if (l < nl) {
+    const uint32_t k = slot_key<EXT>(P, i0 + l, s, t);
+    const uint32_t h = P.slot(i0 + l)[F_HID];
+    id = h & ID_MASK;
+    u = l - div16(l, P.mSub) * nsub;
+    if (k != INF) {
+      const bool hb = (h & HBM_BIT) != 0u;
+      e = hb ? max(k, H) : k;
+      hk = hb ? k : INF;
+    }
+  }
+  const uint32_t hmin = __reduce_min_sync(FULL, hk);
+  uint64_t best = INF64;
+  uint32_t bsl = 0;
+  for (uint32_t v = 0; v < nsub && v < nl; v++) {
+    const uint32_t m = __reduce_min_sync(FULL, u == v ? e : INF);
+    if (m == INF) continue;
+    const uint32_t *sq = P.sub(s, v);
+    const uint32_t E = max(m, sq[Q_AVAIL]), last = sq[Q_LAST];
+    const bool cand = u == v && e <= E;
+    uint32_t key = INF;
+    if (cand) {
+      if (P.policy == GTS_POLICY_GTO) {  // greedy slot, then the oldest warp (CTA id, warp)
+        const uint32_t cs = div16(i0 + l, P.mW);
+        key = (l == last ? 0u : 0x80000000u) | (P.cta(cs)[C_ID] * P.W + (i0 + l - cs * P.W));
+      } else {                            // round-robin after the last slot
+        const uint32_t x = l + per - last - 1u;
+        key = last == NONE ? l : (x >= per ? x - per : x);
+      }
+    }
+    const uint32_t kmin = __reduce_min_sync(FULL, key);
+    const uint32_t wl = __ffs(__ballot_sync(FULL, cand && key == kmin)) - 1;
+    const uint64_t val = pack(E, __shfl_sync(FULL, id, wl));
+    if (val < best) {
+      best = val;
+      bsl = i0 + wl;
+    }
+  }
+  if (lane == 0) {
+    uint32_t *o = P.smrec(s);
+    o[0] = (uint32_t)best;
+    o[1] = (uint32_t)(best >> 32);
+    o[2] = bsl;
+    o[3] = hmin;
+  }
+}
+
 // Warp-parallel: the keys of SM s's heads at cycle t and the SM's summary
 // record.  All lanes call it.
 template <bool EXT>
 __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane) {
   if (EXT && P.L.nsub) {
-    if (lane == 0) rescan_sm_sub<EXT>(P, s, t, H);
+    if (P.L.per <= 32u) rescan_sm_sub_warp<EXT>(P, s, t, H, lane);
+    else if (lane == 0) rescan_sm_sub<EXT>(P, s, t, H);
     __syncwarp();
     return;
   }
