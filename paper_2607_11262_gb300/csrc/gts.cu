@@ -971,6 +971,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       // atomics; into scratch counters by lane 0 (which also reads them later)
       uint32_t adj_cnt = 0, adj_rdy = 0;
       bool cross_touch = false;
+      uint32_t xs = NONE;  // SM of the head in another CTA slot this lane released into (one round only)
       for (uint32_t base = 0; base < deg; base += 32) {
         if (base) ew = (base + lane < deg) ? g.succ[sb + base + lane] : make_uint2(NONE, 0);
         const bool mine = base + lane < deg;
@@ -1004,6 +1005,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
               atomicMax(&ts[F_RDY], rel);
               to_head = true;
               cross = tcs != cs;
+              if (EXT && cross) xs = div16(tcs, P.mCps);
             }
           }
         }
@@ -1029,13 +1031,57 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       set_head(P, i, nx, rn, qn, cn, adj_cnt, adj_rdy);
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
-      if (cross_touch) {  // a release reached a head of another CTA: recompute everything
+      if (EXT && cross_touch && deg <= 32u) {  // releases reached heads of other CTAs: their SMs and this one
+        refresh_sm<EXT>(P, sm, t, C.H, lane);
+        bool own = (uint32_t)lane == (sm & 31u);
+        uint32_t xm = __ballot_sync(FULL, xs != NONE && xs != sm);
+        uint32_t done = sm;
+        while (xm) {
+          const int j = __ffs(xm) - 1;
+          xm &= xm - 1;
+          const uint32_t s2 = __shfl_sync(FULL, xs, j);
+          if (s2 == done) continue;
+          done = s2;
+          refresh_sm<EXT>(P, s2, t, C.H, lane);
+          own |= (uint32_t)lane == (s2 & 31u);
+        }
+        if (C.H != prevH) {  // and the SMs whose HBM heads the new horizon overtakes
+          for (uint32_t s = lane; s < P.L.NS; s += 32) {
+            if (P.smrec(s)[3] < C.H) {
+              rescan_sm_lane<EXT>(P, s, t, C.H);
+              own = true;
+            }
+          }
+        }
+        if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
+          const uint32_t g0 = div16(sm, P.mCsms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
+          for (uint32_t s = g0 + lane; s < g1; s += 32) rescan_sm_lane<EXT>(P, s, t, C.H);
+          __syncwarp();
+          for (uint32_t s = g0; s < g1; s++) own |= (s & 31u) == (uint32_t)lane;
+        }
+        __syncwarp();
+        if (own) b = lane_best(P, lane, bsl);
+      } else if (cross_touch) {  // a node with many successors: recompute everything
         for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane<EXT>(P, s, t, C.H);
         __syncwarp();
         b = lane_best(P, lane, bsl);
       } else {
         refresh_sm<EXT>(P, sm, t, C.H, lane);
-        if (C.H != prevH) {
+        if (C.H != prevH && P.L.per >= 8u && !(EXT && P.L.nsub)) {
+          // SMs of many slots: one SM at a time, a slot per lane
+          bool own = (uint32_t)lane == (sm & 31u);
+          for (uint32_t s0 = 0; s0 < P.L.NS; s0 += 32) {
+            const uint32_t s = s0 + lane;
+            uint32_t xm = __ballot_sync(FULL, s < P.L.NS && s != sm && P.smrec(s)[3] < C.H);
+            while (xm) {
+              const uint32_t s2 = s0 + __ffs(xm) - 1;
+              xm &= xm - 1;
+              refresh_sm<EXT>(P, s2, t, C.H, lane);
+              own |= (uint32_t)lane == (s2 & 31u);
+            }
+          }
+          if (own) b = lane_best(P, lane, bsl);
+        } else if (C.H != prevH) {
           // SMs whose HBM heads H overtakes change their effective cycles
           bool any = false;
           for (uint32_t s = lane; s < P.L.NS; s += 32) {
