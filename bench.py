@@ -63,8 +63,46 @@ def profiled(path, name):
     return f if f.get("source_sha256_16") == source_hash() and name in f.get("applies_to", []) else None
 
 
+def code_tokens(text):
+    """C/C++/CUDA source with comments removed and whitespace runs collapsed
+    (string and character literals kept), so that a comment edit keeps the
+    hash and any change to the code changes it."""
+    out, i, n = [], 0, len(text)
+
+    def space():
+        if out and out[-1] != " ":
+            out.append(" ")
+
+    while i < n:
+        c = text[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and text[j] != c:
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        elif text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+            space()
+        elif c.isspace():
+            j = i
+            while j < n and text[j].isspace():
+                j += 1
+            space()
+            i = j
+        else:
+            out.append(c)
+            i += 1
+    return "".join(out).strip()
+
+
 def source_hash():
-    return hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()[:16]
+    """First 16 hex digits of the SHA-256 of the kernel source's code (comments excluded)."""
+    return hashlib.sha256(code_tokens(open(KERNEL_SRC).read()).encode()).hexdigest()[:16]
 
 
 class Clocks:

@@ -3,7 +3,7 @@
 // One warp simulates one design point (one hardware parameter row) of the
 // graph-driven simulation backend (Section 5).  The warp keeps in shared
 // memory the event frontier -- the head node of every logical warp stream of
-// every resident CTA -- with a cached issue key per head, the per-SM unit
+// every resident CTA -- with each head's release state, the per-SM unit
 // servers, the global HBM servers, the CTA slots, and one summary per
 // simulated SM; it advances the schedule with warp min-reductions.  The tile
 // graph is shared read-only by all points.  Per point, a global scratch row
@@ -24,7 +24,10 @@
 //    minimum over them in registers; the warp takes the minimum over lanes
 //    with two __reduce_min_sync.  After an issue the issuing SM's keys and
 //    summary are recomputed warp-parallel, then its owner lane's minimum;
-//    when H moves, the SMs whose HBM heads it overtakes are recomputed.
+//    when H moves, the SMs whose HBM heads it overtakes are recomputed (each
+//    lane its own SMs, or one SM at a time a slot per lane when SMs hold 8
+//    slots or more).  A release into a head of another CTA recomputes every
+//    SM (the extended instance: the SMs it reached).
 //  * The issue itself runs in every lane on broadcast values (no divergence);
 //    only global atomics and scratch-counter reads are lane 0's.
 //  * Dependency release (Section 5.1).  An issued node releases each
@@ -38,7 +41,8 @@
 //    lanes, fence first.
 //  * Occupancy ceil(work / rate) uses exact division by invariant integers
 //    (Lemire, Kaser, Kurz 2019: floor(n/d) = floor(ceil(2^64/d) * n / 2^64)
-//    for 32-bit n and d), with the per-point constants computed once.
+//    for 32-bit n and d), with the per-point constants computed once; slot,
+//    CTA-slot and SM indices (< 2^16) use the 32-bit form of the same method.
 //  * Server identity is unobservable, so "take any free server" takes the
 //    first free one.
 //  * Every loop is bounded: the per-point step count is capped by
