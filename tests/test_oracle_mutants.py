@@ -9,8 +9,6 @@ import ctypes
 import os
 import subprocess
 
-import pytest
-
 from oracle import run
 from paper_2607_11262_gb300 import workloads as W
 from tests import test_oracle_pins as PINS
