@@ -61,3 +61,43 @@ def test_oracle_builds_and_is_separate():
     for f in ("gts.py", "build.py", "workloads.py"):
         txt = open(os.path.join(ROOT, "paper_2607_11262_gb300", f)).read()
         assert not re.search(r"^\s*(from|import)\s+oracle", txt, flags=re.M), f
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include "gts.h"
+
+int main(void) {
+  /* host-only calls: sizes and the error text need no GPU */
+  printf("%zu %zu %zu\n", gts_graph_workspace_bytes(10, 12, 2, 3, 1), gts_graph_workspace_bytes(10, 12, 2, 200, 1),
+         gts_template_workspace_bytes(2, 20, 40, 50, 4, 3, 1));
+  printf("%d %d\n", gts_graph_create(NULL, NULL, NULL), gts_last_error() != NULL);
+  return 0;
+}
+"""
+
+
+def test_header_is_plain_c_and_a_c_client_links(lib):
+    # a C99 program (pedantic, warnings as errors) includes the header, links
+    # libgts and gets the binding's answers from the host-only calls
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no C compiler")
+    out_dir = os.path.join(os.path.dirname(B.LIB), "c_client")
+    os.makedirs(out_dir, exist_ok=True)
+    src = os.path.join(out_dir, "client.c")
+    exe = os.path.join(out_dir, f"client_{os.getpid()}")
+    with open(src, "w") as f:
+        f.write(C_CLIENT)
+    lib_dir = os.path.dirname(B.LIB)
+    subprocess.check_call(["gcc", "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", os.path.join(ROOT, "include"),
+                           "-o", exe, src, os.path.join(lib_dir, os.path.basename(B.LIB)), f"-Wl,-rpath,{lib_dir}"])
+    try:
+        got = subprocess.run([exe], capture_output=True, text=True, check=True).stdout.split()
+    finally:
+        os.remove(exe)
+    want = [gts.gts_graph_workspace_bytes(10, 12, 2, 3, 1), gts.gts_graph_workspace_bytes(10, 12, 2, 200, 1),
+            gts.gts_template_workspace_bytes(2, 20, 40, 50, 4, 3, 1)]
+    assert [int(x) for x in got[:3]] == want
+    assert int(got[3]) == gts.GTS_ERR_INVALID_ARG and got[4] == "1"
