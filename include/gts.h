@@ -329,7 +329,9 @@ size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint3
  * unspecified.  The digest is sum over v of splitmix64-finalise(
  * (v << 32 | (uint32)start) ^ ((uint64)(uint32)finish * 0x9E3779B97F4A7C15)) mod 2^64.
  * d_scratch (16-byte aligned, scratch_bytes long) is required; see
- * gts_scratch_bytes.  Enqueues on `stream` and returns; *out (may be NULL)
+ * gts_scratch_bytes.  Every other device pointer is aligned to its element
+ * type, as C requires of typed pointers (4 bytes for the int32 arrays, 8 for
+ * d_digest and d_busy); d_busy's alignment is checked (INVALID_ARG).  Enqueues on `stream` and returns; *out (may be NULL)
  * remembers the arrays for gts_read_results.  Errors: INVALID_ARG, NOMEM
  * (scratch smaller than one row), CUDA.
  */
