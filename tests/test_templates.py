@@ -48,3 +48,42 @@ def test_template_csr_is_sorted_and_local():
             succ = ts.col[ts.row_ptr[u]:ts.row_ptr[u + 1]].astype(np.int64)
             assert np.all(np.diff(succ) >= 0)
             assert np.all((succ > u) & (succ < off[t + 1]))
+
+
+def _random_template(rng, warps):
+    t = W.CtaTemplate(warps)
+    n = int(rng.integers(0, 12))
+    for _ in range(n):
+        t.node(int(rng.integers(0, 7)), int(rng.integers(0, warps)), int(rng.integers(0, 5000)), int(rng.integers(0, 9)))
+    for v in range(1, n):
+        for u in rng.choice(v, size=min(v, int(rng.integers(0, 3))), replace=False):
+            t.edge(int(u), v, int(rng.integers(0, 2)))
+    return t
+
+
+def _by_hand(name, warps, tpls, ct, ck):
+    """The logical graph written out CTA by CTA: CTA c's copy of its template
+    takes the next block of ids, edges shifted by that block's base."""
+    typ, wp, wk, lx, cta, src, dst, kind = [], [], [], [], [], [], [], []
+    for c, t in enumerate(ct):
+        tp = tpls[t]
+        base = len(typ)
+        for u in range(len(tp)):
+            typ.append(tp.t[u]); wp.append(tp.w[u]); wk.append(tp.wk[u]); lx.append(tp.lx[u]); cta.append(c)
+        for u, v, k in zip(tp.es, tp.ed, tp.ek):
+            src.append(base + u); dst.append(base + v); kind.append(k)
+    return W.from_edges(name, warps, typ, wp, cta, wk, lx, ck, src, dst, kind)
+
+
+def test_random_template_sets_expand_to_the_hand_built_graph():
+    rng = np.random.default_rng(77)
+    for trial in range(60):
+        warps = int(rng.integers(1, 5))
+        tpls = [_random_template(rng, warps) for _ in range(int(rng.integers(1, 5)))]
+        C = int(rng.integers(1, 12))
+        ct = rng.integers(0, len(tpls), C)
+        ck = np.sort(rng.integers(0, 3, C)).astype(np.uint32)
+        ts = W.template_set(f"r{trial}", warps, tpls, ct, ck)
+        ref = _by_hand(f"r{trial}", warps, tpls, ct, ck)
+        _same(ts.expand(), ref)
+        _same(W.assemble(f"r{trial}", warps, tpls, ct, ck), ref)
