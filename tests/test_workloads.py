@@ -12,7 +12,10 @@ def _contract(g):
     assert np.all(g.warp < g.warps_per_cta)
     assert np.all(g.cta < g.n_ctas)
     assert np.all(np.diff(g.cta_kernel.astype(np.int64)) >= 0)
-    assert np.all(g.type < 7) and np.all(g.ekind <= 1)
+    assert np.all(g.type <= W.DSMEM) and np.all(g.ekind <= 1)
+    if g.tile is not None:
+        named = (g.tile != W.NO_TILE) & ((g.type == W.LOAD) | (g.type == W.STORE))
+        assert np.all(g.tile[named] < g.n_tiles)
     for k in range(g.n_graphs):
         n0, n1 = int(g.node_off[k]), int(g.node_off[k + 1])
         e0, e1 = int(g.row_ptr[n0]), int(g.row_ptr[n1])
@@ -51,3 +54,21 @@ def test_seeded_params_are_reproducible():
     a = W.workload("gemm512").params
     b = W.workload("gemm512").params
     assert np.array_equal(a, b)
+
+
+# published sizes of the configurations (nodes, edges, points); stress is
+# generated at full size only by the GPU tests and the bench (minutes of numpy)
+SIZES = {"gemm512": (2176, 4736, 64), "wsgemm8192": (1581056, 1842144, 4096), "fa_fwd": (1724416, 2232320, 1024),
+         "decoder": (10059776, 11590144, 512)}
+
+
+def test_every_named_workload_keeps_the_contract():
+    for name in ("gemm512", "wsgemm_small", "wsgemm8192", "fa_fwd", "decoder", "pipelines", "noc_fusion", "l2_gemm"):
+        w = W.workload(name)
+        _contract(w.graph)
+        assert w.params.shape[1] == W.NPARAM and w.params.dtype == np.int32, name
+        assert np.all(w.params[:, W.P_GRAPH_INDEX] < w.graph.n_graphs), name
+        if name in SIZES:
+            assert (w.graph.n_nodes, w.graph.n_edges, w.params.shape[0]) == SIZES[name], name
+    assert np.any(W.workload("noc_fusion").graph.type == W.DSMEM)
+    assert W.workload("l2_gemm").graph.n_tiles > 0
