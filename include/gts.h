@@ -158,6 +158,7 @@ typedef int32_t gts_status;
 #define GTS_WANT_DIGEST 2u  /* write d_digest[n_points] */
 #define GTS_WANT_CTA_SM 4u  /* write d_cta_sm [n_points][row_ctas] (-1: never launched) */
 #define GTS_WANT_BUSY   8u  /* write d_busy [n_points][GTS_BUSY_CLASSES] */
+#define GTS_SCRATCH_CLEAN 16u /* d_scratch past its header is all zero (see gts_scratch_bytes) */
 
 /* Busy server-cycles per resource class (Section 5.2 throughput servers):
  * d_busy[q*GTS_BUSY_CLASSES + r] = sum over the point's nodes v that use class
@@ -217,8 +218,9 @@ typedef struct {
 } gts_graph_desc;
 
 /* Bytes of device workspace gts_graph_create needs for a graph of this size
- * (packed node records, successor and predecessor lists, stream heads).
- * Returns 0 when a size is out of range. */
+ * (Section 4.1 tile graph: packed node records, successor lists, the first
+ * node of every (CTA, warp) stream, nodes per CTA).  Returns 0 when a size is
+ * out of range. */
 size_t gts_graph_workspace_bytes(uint32_t n_nodes, uint32_t n_edges, uint32_t n_ctas,
                                  uint32_t warps_per_cta, uint32_t n_graphs);
 
@@ -229,6 +231,8 @@ size_t gts_graph_workspace_bytes(uint32_t n_nodes, uint32_t n_edges, uint32_t n_
  * Errors: INVALID_ARG, INVALID_GRAPH (message names the first offending
  * index), NOMEM (workspace too small), CUDA. */
 gts_status gts_graph_create(const gts_graph_desc *desc, void *stream, gts_graph **out);
+/* Frees the host handle of a graph (Section 4.1); the workspace and the
+ * arrays it borrowed stay the caller's. */
 gts_status gts_graph_destroy(gts_graph *graph);
 
 /*
@@ -280,16 +284,22 @@ size_t gts_template_workspace_bytes(uint32_t n_templates, uint32_t n_tpl_nodes, 
  * NOMEM (workspace), CUDA. */
 gts_status gts_graph_create_templated(const gts_template_desc *desc, void *stream, gts_graph **out);
 
-/* Registers a table of design points: d_params is [n_points][GTS_NPARAM]
+/* Registers a table of design points (one hardware description per point:
+ * the Section 5.2 throughput and latency parameters, with the meanings and
+ * H100 / A100 / B200 values of Section 6.1, Table "GPU configurations used in
+ * evaluation"; fields listed above): d_params is [n_points][GTS_NPARAM]
  * int32 on the device, borrowed by *out.  Copies it to the host to size the
  * per-warp on-chip state of each row; waits for `stream`.  Rows that break the
  * parameter rules are not an error here: gts_simulate_batch reports them as
  * GTS_ERR_INVALID_PARAMS in d_status.  Errors: INVALID_ARG, CUDA. */
 gts_status gts_params_upload(gts_graph *graph, const int32_t *d_params, uint32_t n_points,
                              void *stream, gts_params **out);
+/* Frees the host handle of a parameter table; d_params stays the caller's. */
 gts_status gts_params_destroy(gts_params *params);
 
-/* Attaches a processing order to a parameter table.  Fills d_order (device,
+/* Attaches a processing order to a parameter table.  The paper has no
+ * counterpart: it orders the independent design points of a sweep (the
+ * design-space use of Section 7) over the GPU's warps and changes no result.  Fills d_order (device,
  * [n_points] uint32, caller-owned, borrowed by params) with the point indices
  * sorted by estimated cost, largest first (nodes of the row's graph x (743 +
  * simulated SMs), x 3.5 for rows that need the extended model), and makes
@@ -300,26 +310,38 @@ gts_status gts_params_destroy(gts_params *params);
  * Errors: INVALID_ARG, CUDA. */
 gts_status gts_params_set_order(gts_params *params, uint32_t *d_order, void *stream);
 
-/* Per-point output row lengths: start/finish rows hold gts_row_nodes() entries
- * (the largest graph of the stack), cta_sm rows gts_row_ctas(). */
+/* Per-point output row lengths (the per-node start and finish cycles and the
+ * thread-block placement of Section 5.1): start/finish rows hold
+ * gts_row_nodes() entries (the largest graph of the stack), cta_sm rows
+ * gts_row_ctas(). */
 uint32_t gts_row_nodes(const gts_graph *graph);
 uint32_t gts_row_ctas(const gts_graph *graph);
 
 /* Device scratch gts_simulate_batch wants: GTS_SCRATCH_HEADER_BYTES (the
  * next-point counter of an ordered batch), then one row per concurrently
- * simulated design point -- dependency counters (8 bytes per node of the
- * largest graph, rounded up to 16 bytes) and, for a graph with tiles, one
+ * simulated design point -- dependency counters (Section 5.3 dependency-driven
+ * runtime control: released predecessors and latest release cycle, 8 bytes per
+ * node of the largest graph, rounded up to 16 bytes) and, for a graph with tiles, one
  * 16-byte L2 list record per tile.  Returns the size that lets every resident
  * warp work; a smaller scratch (the header and at least one row) runs fewer
  * points at a time.
- * The kernel clears each row itself; its contents between calls are
- * irrelevant.  Calls sharing one scratch must not overlap on the GPU. */
+ * Every call leaves the rows it used all zero: a node's dependency counters
+ * go back to zero when the node becomes a warp head, and a design point that
+ * stops early (error status) clears what it used.  With GTS_SCRATCH_CLEAN the
+ * caller vouches that the scratch past the header is all zero -- zero-filled
+ * once when allocated and since then passed only to gts_simulate_batch -- and
+ * no row is cleared up front.  Without it each warp clears its row before its
+ * first design point, which writes the whole scratch once per call.  A flag
+ * given for a scratch that is not clean gives wrong results, not a fault.
+ * Calls sharing one scratch must not overlap on the GPU. */
 #define GTS_SCRATCH_HEADER_BYTES 16
 size_t gts_scratch_bytes(const gts_graph *graph, const gts_params *params, uint32_t flags);
 
 /*
  * Simulates design points first_point .. first_point+n_points-1 of `params`
- * on `graph`.  Output arrays are indexed by q = p - first_point:
+ * on `graph`: the graph-driven simulation backend of Section 5 (5.1 execution
+ * flow, 5.2 throughput-oriented hardware model, 5.3 dependency-driven runtime
+ * control), with the semantics stated at the top of this file.  Output arrays are indexed by q = p - first_point:
  *   d_makespan[q], d_status[q]                      (required)
  *   d_start[q*row_nodes + v], d_finish[...]         (GTS_FULL_TRACE; graph-local v)
  *   d_digest[q]                                     (GTS_WANT_DIGEST)
@@ -343,32 +365,40 @@ gts_status gts_simulate_batch(gts_graph *graph, gts_params *params,
                               void *d_scratch, size_t scratch_bytes,
                               void *stream, gts_results **out);
 
-/* Waits for the batch and copies its per-point arrays to the host (any h_*
- * may be NULL; n_points <= the batch's).  Errors: INVALID_ARG, CUDA. */
+/* Waits for the batch and copies its per-point arrays -- the kernel makespan
+ * of each design point (Section 5.1: the cycle the last node completes), its
+ * status and digest -- to the host (any h_* may be NULL; n_points <= the
+ * batch's).  Errors: INVALID_ARG, CUDA. */
 gts_status gts_read_results(gts_results *results, int32_t *h_makespan, int32_t *h_status,
                             uint64_t *h_digest, uint32_t n_points);
+/* Frees a results handle; the device arrays stay the caller's. */
 gts_status gts_results_destroy(gts_results *results);
 
 /*
  * No-allocation variant of gts_simulate_batch.  The paper has no counterpart:
- * it is an interface for callers that cannot allocate device memory at the
- * point of the call -- code running inside a CUDA graph being captured, under
- * an allocator that must not grow, or in a host environment that owns every
- * allocation itself.  Instead of caller scratch it uses one fixed array of
- * GTS_STATIC_SCRATCH_BYTES that lives in the library's own device memory: every
- * GPU that loads the library holds it until the process exits.  The caller
- * still passes every input and output.
- *  - The first call on a device looks up that array's address for the current
- *    device (cudaGetSymbolAddress); make that first call before any stream
- *    capture.  No call allocates or frees device memory.
+ * it is an interface for callers that cannot allocate device memory when they
+ * call it -- a plug-in running inside a host application that owns every
+ * device allocation and hands out no scratch, or a service whose device memory
+ * is fixed at start-up so that its allocator must not grow while requests run.
+ * Instead of caller scratch it uses one fixed array of GTS_STATIC_SCRATCH_BYTES
+ * that lives in the library's own device memory: every GPU that loads the
+ * library holds it until the process exits.  The caller still passes every
+ * input and output.
+ *  - The array's device address is looked up (cudaGetSymbolAddress) on the
+ *    first call in each device context, with that device current, and kept
+ *    with the context's id; a call in a new context (after cudaDeviceReset)
+ *    looks it up again.  The first call may load the library's module on the
+ *    device: make it before any stream capture.  No call allocates or frees
+ *    device memory.
  *  - The scratch header and one row (see gts_scratch_bytes) must fit in
- *    GTS_STATIC_SCRATCH_BYTES, else GTS_ERR_NOMEM: about 4.19 million nodes in
+ *    GTS_STATIC_SCRATCH_BYTES, else GTS_ERR_NOMEM: at most 4,194,302 nodes in
  *    the largest graph without tiles.  Fewer design points then run at a time
  *    than with a large caller scratch (as many as rows fit in the array).
- *  - All calls share the array and the kernel clears each design point's part
- *    before use, so nothing carries over between calls; calls that overlap on
- *    the GPU (other streams, other threads) race on it and must be ordered by
- *    the caller.
+ *  - All calls share the array, which keeps the last call's contents; each
+ *    warp clears its row before its first design point (GTS_SCRATCH_CLEAN is
+ *    ignored here), so nothing carries over between calls.  Calls that overlap
+ *    on the GPU (other streams, other threads) race on it and must be ordered
+ *    by the caller.
  *  - No results handle is returned: read d_makespan / d_status directly.
  * Errors: as gts_simulate_batch, plus NOMEM for a graph too large.
  */
@@ -380,7 +410,8 @@ gts_status gts_simulate_batch_noalloc(gts_graph *graph, gts_params *params,
                                       uint64_t *d_digest, int32_t *d_cta_sm, int64_t *d_busy,
                                       void *stream);
 
-/* Message for the calling thread's last non-OK host-side status ("" if none). */
+/* Message for the calling thread's last non-OK host-side status ("" if none).
+ * Error reporting of this C ABI; the paper has no counterpart. */
 const char *gts_last_error(void);
 
 #ifdef __cplusplus

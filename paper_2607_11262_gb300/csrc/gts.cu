@@ -266,6 +266,10 @@ __device__ __forceinline__ uint2 ld_counters(const uint2 *p) {  // strong load o
   return r;
 }
 
+__device__ __forceinline__ void st_counters_zero(uint2 *p) {  // a counter pair back to (0, 0)
+  asm volatile("st.relaxed.gpu.global.v2.u32 [%0], {%1, %1};" ::"l"(p), "r"(0u) : "memory");
+}
+
 __device__ __forceinline__ uint64_t pack(uint32_t eff, uint32_t id) { return (uint64_t)eff << 32 | id; }
 
 // Warp-wide minimum of a u64 (all lanes get it) and the lowest lane holding it.
@@ -643,6 +647,7 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
         r = g.rec[v];
         q = g.rng[v];
         cc = ld_counters(P.scr + (v - P.n0));
+        if (cc.x | cc.y) st_counters_zero(P.scr + (v - P.n0));  // read once: leave the row clean
       }
       set_head(P, i, v, r, q, cc, 0u, 0u);
     }
@@ -728,6 +733,12 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
   P.W = g.W;
   uint32_t *sp = P.sp;
   const bool want_digest = d_digest != nullptr;
+  // The warp's scratch row is all zero between its points: a node's counter
+  // pair is reset when the node becomes a warp head (after that, releases
+  // reach it in shared memory), and a point that stops early clears the part
+  // it used.  A row is cleared once, before the warp's first point, unless
+  // the caller vouches that the scratch is already clean.
+  bool row_clean = (flags & GTS_SCRATCH_CLEAN) != 0u;
 
   // points: the next one in `order` (a counter in the scratch header), or
   // gw, gw + n_warps, ... without an order
@@ -828,13 +839,11 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       sp[P.L.o_sub + k * SUB_WORDS + Q_AVAIL] = 0u;
       sp[P.L.o_sub + k * SUB_WORDS + Q_LAST] = NONE;
     }
-    {
+    if (!row_clean) {  // the whole row: counters of the largest graph, then the L2 list records
       uint4 *z = reinterpret_cast<uint4 *>(P.scr);
-      const uint32_t nz = nG / 2;
+      const uint32_t nz = ((g.row_nodes + 1u) >> 1) + g.n_tiles;
       for (uint32_t k = lane; k < nz; k += 32) z[k] = make_uint4(0, 0, 0, 0);
-      if ((nG & 1u) && lane == 0) P.scr[nG - 1] = make_uint2(0, 0);
-      if (l2on)
-        for (uint32_t k = lane; k < g.n_tiles; k += 32) l2t[k] = make_uint4(0, 0, 0, 0);
+      row_clean = true;
     }
     if (cta_sm_row)
       for (uint32_t c = lane; c < CG; c += 32) cta_sm_row[c] = -1;
@@ -1030,6 +1039,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         }
       }
       __syncwarp();
+      if (lane == 0 && (cn.x | cn.y)) st_counters_zero(P.scr + (nx - P.n0));  // read once: leave the row clean
       cn.x = __shfl_sync(FULL, cn.x, 0);  // the next head's counters (its scratch row is not released into above)
       cn.y = __shfl_sync(FULL, cn.y, 0);
       set_head(P, i, nx, rn, qn, cn, adj_cnt, adj_rdy);
@@ -1117,6 +1127,18 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         }
       }
     }
+    // leave the row clean: a point that stopped early may hold counters of
+    // nodes that never became heads; the L2 list records are always used
+    if (status != GTS_OK || l2on) {
+      __threadfence();  // lane 0's releases and list updates come before the clears
+      __syncwarp();
+      uint4 *z = reinterpret_cast<uint4 *>(P.scr);
+      const uint32_t nz = status != GTS_OK ? (nG + 1u) >> 1 : 0u;
+      for (uint32_t k = lane; k < nz; k += 32) z[k] = make_uint4(0, 0, 0, 0);
+      if (l2on)
+        for (uint32_t k = lane; k < g.n_tiles; k += 32) l2t[k] = make_uint4(0, 0, 0, 0);
+    }
+    __threadfence();
     if (lane == 0) {
       d_status[q] = status;
       d_makespan[q] = status == GTS_OK ? mk : 0;
@@ -1631,8 +1653,10 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
       pl.wpb = wpb;
     }
   }
-  pl.smem = pl.wpb * bytes;
   uint64_t warps = (uint64_t)std::max(best_w, 1u) * sms;
+  // a batch smaller than one wave: blocks small enough that every SM gets one
+  // before any gets two (the block scheduler fills SMs breadth first)
+  if (np < warps) pl.wpb = std::max(1u, std::min(pl.wpb, np / (uint32_t)sms));
   warps = std::min<uint64_t>(warps, np);
   if (limit_by_scratch) {
     const uint64_t row = scratch_row_bytes(g);
@@ -1662,7 +1686,7 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
   clear_error();
   if (out) *out = nullptr;
   if (!g || !P || P->graph != g) return fail(GTS_ERR_INVALID_ARG, "null or mismatched graph / params");
-  if (flags & ~(GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM | GTS_WANT_BUSY))
+  if (flags & ~(GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM | GTS_WANT_BUSY | GTS_SCRATCH_CLEAN))
     return fail(GTS_ERR_INVALID_ARG, "unknown flag");
   if ((uint64_t)first_point + n_points > P->n_points) return fail(GTS_ERR_INVALID_ARG, "point range outside the table");
   if (!d_makespan || !d_status) return fail(GTS_ERR_INVALID_ARG, "d_makespan and d_status are required");
@@ -1733,17 +1757,42 @@ gts_status gts_results_destroy(gts_results *r) {
 
 // ----------------------------------------------------------------- no-allocation entry point
 // Scratch for gts_simulate_batch_noalloc: a fixed array in the library's own
-// device memory, created when the module loads on a device and held until the
-// process exits.  In host code the symbol is only a handle; its device address
-// comes from cudaGetSymbolAddress, resolved once per device.
+// device memory, created when the module loads in a device's context and held
+// until the process exits.  In host code the symbol is only a handle; its
+// device address comes from cudaGetSymbolAddress, looked up once per device
+// and context: the context's process-unique id (cuCtxGetId) is kept with the
+// address, so a call after cudaDeviceReset (a new context, the module loaded
+// anew) looks the address up again instead of using the old one.
 static __device__ __align__(256) uint2 g_static_scratch[GTS_STATIC_SCRATCH_BYTES / sizeof(uint2)];
 
 namespace {
 constexpr int MAX_DEVICES = 64;
-void *g_static_ptr[MAX_DEVICES];
+struct StaticScratch {
+  unsigned long long ctx_id;
+  void *ptr;
+};
+StaticScratch g_static[MAX_DEVICES];
 std::atomic<int> g_static_lock{0};
+typedef int (*ctx_get_id_fn)(void *ctx, unsigned long long *id);  // CUresult cuCtxGetId(CUcontext, ...)
+ctx_get_id_fn g_ctx_get_id = nullptr;
 
-// Address of this device's static scratch (set-up on the first call per device).
+// Id of the current context, or 0 when none is current yet.
+gts_status current_ctx_id(unsigned long long *id) {
+  *id = 0;
+  if (!g_ctx_get_id) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    const cudaError_t e = cudaGetDriverEntryPointByVersion("cuCtxGetId", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+      return fail(GTS_ERR_CUDA, "simulate_noalloc: driver entry point cuCtxGetId unavailable");
+    g_ctx_get_id = (ctx_get_id_fn)fn;
+  }
+  if (g_ctx_get_id(nullptr, id) != 0) *id = 0;
+  return GTS_OK;
+}
+
+// Address of the static scratch in the current device's context (set-up on
+// the first call in each device context).
 gts_status static_scratch(void **out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -1751,14 +1800,20 @@ gts_status static_scratch(void **out) {
   if (dev < 0 || dev >= MAX_DEVICES) return fail(GTS_ERR_UNSUPPORTED, "simulate_noalloc: device ordinal above 63");
   while (g_static_lock.exchange(1, std::memory_order_acquire)) {
   }
-  gts_status st = GTS_OK;
-  if (!g_static_ptr[dev]) {
+  unsigned long long id = 0;
+  gts_status st = current_ctx_id(&id);
+  if (st == GTS_OK && (id == 0 || g_static[dev].ctx_id != id || !g_static[dev].ptr)) {
     void *p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_static_scratch);
-    if (e != cudaSuccess) st = cuda_fail(e, "simulate_noalloc: static scratch address");
-    else g_static_ptr[dev] = p;
+    e = cudaGetSymbolAddress(&p, g_static_scratch);  // makes the device's context current if none was
+    if (e != cudaSuccess) {
+      st = cuda_fail(e, "simulate_noalloc: static scratch address");
+    } else {
+      if (id == 0) current_ctx_id(&id);
+      g_static[dev].ctx_id = id;
+      g_static[dev].ptr = p;
+    }
   }
-  *out = g_static_ptr[dev];
+  *out = g_static[dev].ptr;
   g_static_lock.store(0, std::memory_order_release);
   return st;
 }
@@ -1778,6 +1833,8 @@ gts_status gts_simulate_batch_noalloc(gts_graph *g, gts_params *P, uint32_t firs
   void *scr = nullptr;
   gts_status st = static_scratch(&scr);
   if (st != GTS_OK) return st;
+  // the shared array is cleared row by row before use (never vouched clean)
+  flags &= ~GTS_SCRATCH_CLEAN;
   return gts_simulate_batch(g, P, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status, d_digest,
                             d_cta_sm, d_busy, scr, GTS_STATIC_SCRATCH_BYTES, stream, nullptr);
 }

@@ -33,6 +33,7 @@ GTS_FULL_TRACE = 1
 GTS_WANT_DIGEST = 2
 GTS_WANT_CTA_SM = 4
 GTS_WANT_BUSY = 8
+GTS_SCRATCH_CLEAN = 16
 
 GTS_BUSY_CLASSES = 9
 (GTS_BUSY_TENSOR, GTS_BUSY_TMA, GTS_BUSY_LSU, GTS_BUSY_ALU, GTS_BUSY_BAR, GTS_BUSY_HBM, GTS_BUSY_NOC,
@@ -401,6 +402,15 @@ def _ptr(t):
     return 0 if t is None else t.data_ptr()
 
 
+def alloc_scratch(dgraph: DeviceGraph, dparams: DeviceParams, flags=0, stream=None):
+    """A zero-filled scratch of gts_scratch_bytes; pass it to ``simulate`` with
+    GTS_SCRATCH_CLEAN in the flags, call after call (libgts leaves it clean)."""
+    import torch
+    nb = gts_scratch_bytes(dgraph.handle, dparams.handle, flags)
+    with torch.cuda.stream(stream) if stream is not None else _null():
+        return torch.zeros(max(nb, 16), dtype=torch.uint8, device=dgraph.workspace.device)
+
+
 def simulate(dgraph: DeviceGraph, dparams: DeviceParams, first_point=0, n_points=None,
              flags=GTS_FULL_TRACE | GTS_WANT_DIGEST | GTS_WANT_CTA_SM, out: BatchOutput = None,
              scratch=None, stream=None) -> BatchOutput:
@@ -410,9 +420,10 @@ def simulate(dgraph: DeviceGraph, dparams: DeviceParams, first_point=0, n_points
         n_points = dparams.n_points - first_point
     if out is None:
         out = alloc_outputs(dgraph, n_points, flags)
-    if scratch is None:
+    if scratch is None:  # zero-filled, so the kernel need not clear it (GTS_SCRATCH_CLEAN)
         nb = gts_scratch_bytes(dgraph.handle, dparams.handle, flags)
-        scratch = torch.empty(max(nb, 16), dtype=torch.uint8, device=dgraph.workspace.device)
+        scratch = torch.zeros(max(nb, 16), dtype=torch.uint8, device=dgraph.workspace.device)
+        flags |= GTS_SCRATCH_CLEAN
     gts_simulate_batch(dgraph.handle, dparams.handle, first_point, n_points, flags, _ptr(out.start),
                        _ptr(out.finish), _ptr(out.makespan), _ptr(out.status), _ptr(out.digest),
                        _ptr(out.cta_sm), _ptr(out.busy), _ptr(scratch), 0 if scratch is None else scratch.numel(),

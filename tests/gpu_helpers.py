@@ -20,6 +20,28 @@ def digest(start, finish):
         return int(np.sum(z, dtype=np.uint64))
 
 
+def _mix(z):
+    with np.errstate(over="ignore"):
+        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)
+        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
+        return z ^ (z >> np.uint64(31))
+
+
+def aux_digest(cta_sm, busy):
+    """A host-side digest of one point's CTA placement and busy counters:
+    sum over c of mix(c << 32 | cta_sm[c]) plus sum over k of mix((k + 1) << 56 ^ busy[k]),
+    mod 2^64 (mix = the splitmix64 finaliser).  Used only to compare the GPU's
+    outputs with stored oracle results."""
+    c = np.arange(len(cta_sm), dtype=np.uint64)
+    s = np.asarray(cta_sm, np.int64).astype(np.uint32).astype(np.uint64)
+    k = np.arange(len(busy), dtype=np.uint64) + np.uint64(1)
+    b = np.asarray(busy, np.int64).astype(np.uint64)
+    with np.errstate(over="ignore"):
+        t1 = np.sum(_mix((c << np.uint64(32)) | s), dtype=np.uint64)
+        t2 = np.sum(_mix((k << np.uint64(56)) ^ b), dtype=np.uint64)
+        return int((int(t1) + int(t2)) & MASK64)
+
+
 def run_gpu(graph, params, flags=None, first_point=0, n_points=None):
     import torch
 

@@ -1,7 +1,9 @@
 """gts_simulate_batch_noalloc -- the entry point for callers that cannot
-allocate device memory when they call (inside stream capture, under a fixed
-allocator, or where the host owns every allocation) -- gives the same results
-as gts_simulate_batch with caller scratch, call after call.
+allocate device memory when they call it (a plug-in inside a host application
+that owns every device allocation, or a service whose device memory is fixed
+at start-up so its allocator must not grow) -- gives the same results as
+gts_simulate_batch with caller scratch, call after call, and allocates
+nothing.
 
 This file is collected last on purpose: it shares the library's static scratch
 with nothing else and must pass alone in a fresh process or after the rest.
@@ -87,15 +89,49 @@ def test_noalloc_partial_range_and_too_large(gts_mod):
     part = _noalloc(gts, dg, dp, out, first=10, n=20)
     for k in part:
         assert np.array_equal(part[k], ref[k][10:30]), k
-    # a graph with more nodes than the static array holds is refused
-    n = gts.GTS_STATIC_SCRATCH_BYTES // 8 + 2
-    big = W.from_edges("big", 1, np.full(n, W.NOP, np.uint8), np.zeros(n, np.uint16), np.zeros(n, np.uint32),
-                       np.zeros(n, np.uint32), np.zeros(n, np.uint32), np.zeros(1, np.uint32), [], [], [])
-    dgb = gts.DeviceGraph(big)
-    dpb = gts.DeviceParams(dgb, TG.unit_params()[None, :])
-    outb = gts.alloc_outputs(dgb, 1, 0)
-    with pytest.raises(gts.GtsError) as e:
-        gts.gts_simulate_batch_noalloc(dgb.handle, dpb.handle, 0, 1, 0, 0, 0, outb.makespan.data_ptr(),
-                                       outb.status.data_ptr(), 0, 0, 0, 0)
-    assert e.value.status == gts.GTS_ERR_NOMEM
-    assert "static scratch" in gts.gts_last_error()
+
+
+def _nop_graph(n):
+    return W.from_edges("nops", 1, np.full(n, W.NOP, np.uint8), np.zeros(n, np.uint16), np.zeros(n, np.uint32),
+                        np.zeros(n, np.uint32), np.zeros(n, np.uint32), np.zeros(1, np.uint32), [], [], [])
+
+
+def test_noalloc_size_limit_exact(gts_mod):
+    """The header (16 B) and one row (8 B per node, rounded to an even count)
+    must fit in GTS_STATIC_SCRATCH_BYTES: 4,194,302 nodes do, 4,194,303 not."""
+    gts = gts_mod
+    limit = (gts.GTS_STATIC_SCRATCH_BYTES - gts.GTS_SCRATCH_HEADER_BYTES) // 8
+    assert limit == 4_194_302
+    for n, ok in ((limit, True), (limit + 1, False)):
+        dg = gts.DeviceGraph(_nop_graph(n))
+        dp = gts.DeviceParams(dg, TG.unit_params()[None, :])
+        out = gts.alloc_outputs(dg, 1, 0)
+        call = lambda: gts.gts_simulate_batch_noalloc(dg.handle, dp.handle, 0, 0, 0, 0, 0,  # noqa: E731
+                                                      out.makespan.data_ptr(), out.status.data_ptr(), 0, 0, 0, 0)
+        if ok:
+            call()  # size accepted (no point requested, so nothing runs)
+        else:
+            with pytest.raises(gts.GtsError) as e:
+                call()
+            assert e.value.status == gts.GTS_ERR_NOMEM
+            assert "static scratch" in gts.gts_last_error()
+        dp.close()
+        dg.close()
+
+
+def test_noalloc_allocates_no_device_memory(gts_mod):
+    """After a first call (which loads the module and looks up the array), a
+    call leaves the device's free memory unchanged."""
+    import torch
+    gts = gts_mod
+    w = W.workload("gemm512")
+    dg = gts.DeviceGraph(w.graph)
+    dp = gts.DeviceParams(dg, w.params)
+    out = gts.alloc_outputs(dg, dp.n_points, FLAGS)
+    first = _noalloc(gts, dg, dp, out)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    again = _noalloc(gts, dg, dp, out)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    _same(again, first)
