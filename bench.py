@@ -361,6 +361,7 @@ def main():
     ap.add_argument("--policy", default="lowest_id", choices=sorted(POLICIES))
     ap.add_argument("--subpartitions", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (e2e is then null)")
     ap.add_argument("--ref-seconds", type=float, default=15.0)
     ap.add_argument("--ref-points-per-core", type=int, default=1)
     args = ap.parse_args()
@@ -422,7 +423,7 @@ def main():
 
     # ---- e2e: host buffers through the C ABI, copies inside the timed region
     e2e = None
-    if rank == 0 or ws > 1:
+    if (rank == 0 or ws > 1) and not args.no_e2e:
         from paper_2607_11262_gb300 import workloads as W
         templates = W.workload(args.workload, templated=True).graph if args.workload in W.TEMPLATED else None
         e2e = measure_e2e(g, w.params, gts, stream, templates=templates)

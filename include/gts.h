@@ -210,7 +210,7 @@ typedef struct {
   const uint32_t *work;             /* [n_nodes] bytes / FMAs / ops */
   const uint32_t *lat_extra;        /* [n_nodes] extra latency, cycles */
   const uint32_t *cta_kernel;       /* [n_ctas] */
-  void *workspace;                  /* device, >= gts_graph_workspace_bytes(...) */
+  void *workspace;                  /* device, 16-byte aligned, >= gts_graph_workspace_bytes(...) */
   size_t workspace_bytes;
   const uint32_t *tile;             /* [n_nodes] tile a LOAD/STORE reads or writes, < n_tiles, or
                                        0xFFFFFFFF (none); ignored on other types; NULL: no tiles */
@@ -219,17 +219,22 @@ typedef struct {
 
 /* Bytes of device workspace gts_graph_create needs for a graph of this size
  * (Section 4.1 tile graph: packed node records, successor lists, the first
- * node of every (CTA, warp) stream, nodes per CTA).  Returns 0 when a size is
- * out of range. */
+ * node of every (CTA, warp) stream, nodes per CTA, and the check's status
+ * words and per-CTA temporaries, zero once the call returns).  Returns 0 when
+ * a size is out of range. */
 size_t gts_graph_workspace_bytes(uint32_t n_nodes, uint32_t n_edges, uint32_t n_ctas,
                                  uint32_t warps_per_cta, uint32_t n_graphs);
 
 /* Checks the graph contract and builds the derived device arrays into
- * desc->workspace (Section 4.1 graph, Section 5.1 per-TB streams).  Copies the
- * graph to the host to check and pack it, then back; waits for `stream`.
- * *out borrows desc->cta_kernel and desc->workspace.
- * Errors: INVALID_ARG, INVALID_GRAPH (message names the first offending
- * index), NOMEM (workspace too small), CUDA. */
+ * desc->workspace (Section 4.1 graph, Section 5.1 per-TB streams), on the
+ * device: the graph never leaves it.  The host reads the graph offsets, the
+ * two ends of row_ptr and a few status words back; graphs whose CTAs
+ * interleave over id spans longer than 32 x n_nodes in total also have their
+ * CTA and warp arrays and node records copied through the host to link the
+ * warp streams.  Waits for `stream`.  *out borrows desc->cta_kernel and
+ * desc->workspace.
+ * Errors: INVALID_ARG, INVALID_GRAPH (message names the check and the lowest
+ * offending index), UNSUPPORTED (in-degree), NOMEM (workspace too small), CUDA. */
 gts_status gts_graph_create(const gts_graph_desc *desc, void *stream, gts_graph **out);
 /* Frees the host handle of a graph (Section 4.1); the workspace and the
  * arrays it borrowed stay the caller's. */
@@ -266,7 +271,7 @@ typedef struct {
   const uint32_t *tpl_lat_extra;   /* [n_tpl_nodes] */
   const uint32_t *cta_template;    /* [n_ctas] */
   const uint32_t *cta_kernel;      /* [n_ctas] */
-  void *workspace;                 /* device, >= gts_template_workspace_bytes(...) */
+  void *workspace;                 /* device, 16-byte aligned, >= gts_template_workspace_bytes(...) */
   size_t workspace_bytes;
 } gts_template_desc;
 

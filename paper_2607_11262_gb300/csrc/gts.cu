@@ -1152,8 +1152,19 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
 size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct WsLayout {
-  size_t rec, rng, succ, first, cnt, noff, coff, total;
+  size_t rec, rng, succ, first, cnt, noff, coff, stat, chi, total;
 };
+
+// Status words of the device-side graph check (GK_* index: first offending
+// node / edge / CTA, NONE if none), then its reductions.
+enum : uint32_t {
+  GK_ROWPTR = 0, GK_TYPE, GK_WARP, GK_CTA, GK_TILE, GK_EDGE, GK_KIND, GK_KERNEL, GK_INDEG, GK_NCHECKS,
+  GK_CLASS = GK_NCHECKS, GK_CROSS,
+  GK_SPAN_LO = 12, GK_SPAN_HI = 13,  // one 64-bit word: 8-byte aligned (the status block is 256-byte aligned)
+  GK_WORDS = 16
+};
+static_assert(GK_CROSS < GK_SPAN_LO && GK_SPAN_LO % 2 == 0 && GK_SPAN_HI == GK_SPAN_LO + 1 && GK_SPAN_HI < GK_WORDS,
+              "the span sum is an aligned 64-bit word after the other status words");
 
 bool ws_layout(uint64_t n, uint64_t m, uint64_t C, uint64_t W, uint64_t G, WsLayout &w) {
   if (n >= 0x7FFFFFFEull || C >= (1ull << 24) || W < 1 || W > MAX_W || G < 1 || G > C + n + 1) return false;
@@ -1165,9 +1176,172 @@ bool ws_layout(uint64_t n, uint64_t m, uint64_t C, uint64_t W, uint64_t G, WsLay
   w.cnt = o; o += align_up(C * 4);
   w.noff = o; o += align_up((G + 1) * 4);
   w.coff = o; o += align_up((G + 1) * 4);
-  w.total = o + 256;
+  o += 256;
+  // used only while gts_graph_create runs, zero afterwards
+  w.stat = o; o += align_up(GK_WORDS * 4);
+  w.chi = o; o += align_up(C * 4);
+  w.total = o;
   return true;
 }
+
+// ---------------------------------------------------------------- device-side graph check and packing
+// Graph of node / CTA x: the g with off[g] <= x < off[g+1] (off non-decreasing, off[0] = 0 <= x < off[G]).
+__device__ __forceinline__ uint32_t graph_of(const uint32_t *off, uint32_t G, uint32_t x) {
+  uint32_t lo = 0, hi = G;  // off[lo] <= x < off[hi]
+  while (hi - lo > 1) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (off[mid] <= x) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
+struct GraphIn {  // the caller's arrays (gts_graph_desc)
+  const uint32_t *row_ptr, *col, *cta, *work, *lx, *kern, *tile;
+  const uint8_t *ek, *ty;
+  const uint16_t *wp;
+  uint32_t n, m, C, W, G, n_tiles;
+};
+
+// Contract checks of the Section 4.1 graph, one thread per node (edges of the
+// node in the same thread).  Records the first offending index per check;
+// touches memory only at indices it has checked.  Also counts in-degrees
+// (into rng[].y), nodes per CTA, the first node of every (CTA, warp) stream
+// and the last node of every CTA, and ORs the unit classes in use and whether
+// an edge crosses CTAs.
+__global__ void k_graph_check(GraphIn in, const uint32_t *noff, const uint32_t *coff, uint32_t *stat, uint4 *rng,
+                              uint32_t *first, uint32_t *cnt, uint32_t *chi) {
+  const uint32_t lane = threadIdx.x & 31u;
+  uint32_t cls_or = 0u, cross = 0u;
+  for (uint32_t v0 = blockIdx.x * blockDim.x; v0 < in.n; v0 += gridDim.x * blockDim.x) {
+    const uint32_t v = v0 + threadIdx.x;
+    if (v < in.n) {
+      const uint32_t g = graph_of(noff, in.G, v);
+      const uint32_t n1 = noff[g + 1], c0 = coff[g], c1 = coff[g + 1];
+      const uint32_t a = in.row_ptr[v], b = in.row_ptr[v + 1];
+      const bool rows_ok = a <= b && b <= in.m;
+      if (!rows_ok) atomicMin(&stat[GK_ROWPTR], v);
+      const uint32_t ty = in.ty[v], wp = in.wp[v], c = in.cta[v];
+      if (ty > GTS_DSMEM) atomicMin(&stat[GK_TYPE], v);
+      else {
+        const uint32_t k = (TYPE_CLASS >> (4 * ty)) & 15u;
+        if (k < RC_N) cls_or |= 1u << k;
+        if (k == RC_DSM) cls_or |= (1u << RC_LSU) | CM_NOC;
+      }
+      if (wp >= in.W) atomicMin(&stat[GK_WARP], v);
+      const bool cta_ok = c >= c0 && c < c1;
+      if (!cta_ok) atomicMin(&stat[GK_CTA], v);
+      if (in.tile && (ty == GTS_LOAD || ty == GTS_STORE) && in.tile[v] != NONE && in.tile[v] >= in.n_tiles)
+        atomicMin(&stat[GK_TILE], v);
+      if (cta_ok) {
+        atomicAdd(&cnt[c], 1u);
+        atomicMax(&chi[c], v);
+        if (wp < in.W) atomicMin(&first[(size_t)c * in.W + wp], v);
+      }
+      if (rows_ok) {
+        for (uint32_t x = a; x < b; x++) {
+          const uint32_t w = in.col[x];
+          if (w <= v || w >= n1) {
+            atomicMin(&stat[GK_EDGE], x);
+          } else {
+            atomicAdd(&rng[w].y, 1u);
+            if (in.cta[w] != c) cross = 1u;
+          }
+          if (in.ek[x] > 1u) atomicMin(&stat[GK_KIND], x);
+        }
+      }
+    }
+  }
+  cls_or = __reduce_or_sync(FULL, cls_or);
+  cross = __reduce_or_sync(FULL, cross);
+  if (lane == 0) {
+    if (cls_or) atomicOr(&stat[GK_CLASS], cls_or);
+    if (cross) atomicOr(&stat[GK_CROSS], 1u);
+  }
+}
+
+// Second pass, after every in-degree and stream head is known: in-degree
+// limit per node, kernel ids non-decreasing within each graph per CTA, and
+// the sum over CTAs of their id span (last - first node + 1), the work of the
+// stream-link pass below.
+__global__ void k_graph_check2(GraphIn in, const uint32_t *coff, uint32_t *stat, const uint4 *rng,
+                               const uint32_t *first, const uint32_t *cnt, const uint32_t *chi) {
+  unsigned long long span = 0ull;
+  const uint32_t N = max(in.n, in.C);
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < N; i += gridDim.x * blockDim.x) {
+    if (i < in.n && rng[i].y > MAX_INDEG) atomicMin(&stat[GK_INDEG], i);
+    if (i < in.C) {
+      if (i > 0 && graph_of(coff, in.G, i) == graph_of(coff, in.G, i - 1) && in.kern[i] < in.kern[i - 1])
+        atomicMin(&stat[GK_KERNEL], i);
+      if (cnt[i]) {
+        uint32_t lo = NONE;
+        for (uint32_t w = 0; w < in.W; w++) lo = min(lo, first[(size_t)i * in.W + w]);
+        span += (unsigned long long)(chi[i] - lo) + 1ull;
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) span += __shfl_down_sync(FULL, span, o);
+  if ((threadIdx.x & 31u) == 0 && span) {
+    unsigned long long *s64 = reinterpret_cast<unsigned long long *>(stat + GK_SPAN_LO);
+    atomicAdd(s64, span);
+  }
+}
+
+// Packed node records, ranges and successor entries (the layout k_simulate
+// reads), one thread per node.  The stream link (rec.z) is filled by
+// k_graph_streams.
+__global__ void k_graph_pack(GraphIn in, uint4 *rec, uint4 *rng, uint2 *succ) {
+  for (uint32_t v = blockIdx.x * blockDim.x + threadIdx.x; v < in.n; v += gridDim.x * blockDim.x) {
+    const uint32_t a = in.row_ptr[v], b = in.row_ptr[v + 1], ty = in.ty[v];
+    const uint32_t indeg = rng[v].y;
+    const bool tiled = in.tile && in.tile[v] != NONE && (ty == GTS_LOAD || ty == GTS_STORE);
+    rec[v] = make_uint4(in.work[v], in.lx[v], NONE, ty | (indeg << 4));
+    rng[v] = make_uint4(tiled ? in.tile[v] + 1u : 0u, 0u, a, b);
+    for (uint32_t x = a; x < b; x++) {
+      const uint32_t w = in.col[x];
+      succ[x] = make_uint2(w, (uint32_t)in.ek[x] | ((uint32_t)in.wp[w] << 1) | (in.cta[w] << 8));
+    }
+  }
+}
+
+// Program order of every (CTA, warp) stream (Section 5.1: each warp issues its
+// nodes in ascending id): rec[v].z = the next node of v's stream.  One warp
+// per CTA walks the CTA's id span downwards, 32 ids at a time; lanes holding
+// nodes of the CTA group by warp (match), each takes the next higher lane of
+// its group, and the group's lowest lane leaves its id for the chunk below.
+__global__ void k_graph_streams(GraphIn in, const uint32_t *first, const uint32_t *cnt, const uint32_t *chi,
+                                uint4 *rec) {
+  extern __shared__ uint32_t carry_all[];  // W per warp
+  const uint32_t lane = threadIdx.x & 31u, wib = threadIdx.x >> 5, wpb = blockDim.x >> 5;
+  uint32_t *carry = carry_all + wib * in.W;
+  for (uint32_t c = blockIdx.x * wpb + wib; c < in.C; c += gridDim.x * wpb) {
+    if (cnt[c] == 0u) continue;
+    uint32_t lo = NONE;
+    for (uint32_t w = lane; w < in.W; w += 32) {
+      carry[w] = NONE;
+      lo = min(lo, first[(size_t)c * in.W + w]);
+    }
+    lo = __reduce_min_sync(FULL, lo);
+    const uint32_t hi = chi[c];
+    __syncwarp();
+    for (uint32_t top = hi + 1u; top > lo;) {
+      const uint32_t base = top - lo >= 32u ? top - 32u : lo;
+      const uint32_t v = base + lane;
+      const bool mine = v < top && in.cta[v] == c;
+      const uint32_t key = mine ? (uint32_t)in.wp[v] : NONE;
+      const uint32_t peers = __match_any_sync(FULL, key);
+      if (mine) {
+        const uint32_t higher = peers & ~((2u << lane) - 1u);
+        rec[v].z = higher ? base + (uint32_t)__ffs(higher) - 1u : carry[key];
+      }
+      __syncwarp();
+      if (mine && lane == (uint32_t)__ffs(peers) - 1u) carry[key] = v;
+      __syncwarp();
+      top = base;
+    }
+  }
+}
+
+
 
 template <class T>
 cudaError_t d2h(std::vector<T> &dst, const T *src, size_t count, cudaStream_t s) {
@@ -1316,25 +1490,18 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
   if (G > 1 && (!d->graph_node_off || !d->graph_cta_off))
     return fail(GTS_ERR_INVALID_ARG, "stacked graph needs graph_node_off and graph_cta_off");
   if (!d->workspace) return fail(GTS_ERR_INVALID_ARG, "null workspace");
+  if ((uintptr_t)d->workspace % 16 != 0) return fail(GTS_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
   if (d->workspace_bytes < wl.total)
     return fail(GTS_ERR_NOMEM, "workspace too small: need " + std::to_string(wl.total) + " bytes");
-  cudaStream_t s = (cudaStream_t)stream;
-  std::vector<uint32_t> row_ptr, col, cta, work, lx, kern, noff, coff, tile;
-  std::vector<uint8_t> ek, ty;
-  std::vector<uint16_t> wp;
-  cudaError_t e = cudaSuccess;
   if (d->tile && (d->n_tiles == 0 || d->n_tiles > (1u << 28)))
     return fail(GTS_ERR_INVALID_ARG, "tiles need 1 <= n_tiles <= 2^28");
-  if (e == cudaSuccess && d->tile) e = d2h(tile, d->tile, n, s);
-  if (e == cudaSuccess) e = d2h(row_ptr, d->row_ptr, n + 1, s);
-  if (e == cudaSuccess) e = d2h(col, d->col, m, s);
-  if (e == cudaSuccess) e = d2h(ek, d->ekind, m, s);
-  if (e == cudaSuccess) e = d2h(ty, d->type, n, s);
-  if (e == cudaSuccess) e = d2h(wp, d->warp, n, s);
-  if (e == cudaSuccess) e = d2h(cta, d->cta, n, s);
-  if (e == cudaSuccess) e = d2h(work, d->work, n, s);
-  if (e == cudaSuccess) e = d2h(lx, d->lat_extra, n, s);
-  if (e == cudaSuccess) e = d2h(kern, d->cta_kernel, C, s);
+  cudaStream_t s = (cudaStream_t)stream;
+  char *ws = (char *)d->workspace;
+  // ---- the graph offsets and the ends of row_ptr come to the host (a few words)
+  std::vector<uint32_t> noff, coff, ends;
+  cudaError_t e = d2h(ends, d->row_ptr, 1, s);
+  uint32_t last = 0;
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&last, d->row_ptr + n, 4, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) {
     if (G > 1 || d->graph_node_off) e = d2h(noff, d->graph_node_off, G + 1, s);
     else noff = {0u, (uint32_t)n};
@@ -1344,80 +1511,110 @@ gts_status gts_graph_create(const gts_graph_desc *d, void *stream, gts_graph **o
     else coff = {0u, (uint32_t)C};
   }
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-  if (e != cudaSuccess) return cuda_fail(e, "graph_create: copy to host");
-
-  // ---- contract
+  if (e != cudaSuccess) return cuda_fail(e, "graph_create: copy offsets to host");
   if (noff[0] != 0 || noff[G] != n || coff[0] != 0 || coff[G] != C)
     return fail(GTS_ERR_INVALID_GRAPH, "graph offsets must start at 0 and end at n_nodes / n_ctas");
   for (uint64_t k = 0; k < G; k++)
     if (noff[k + 1] < noff[k] || coff[k + 1] < coff[k])
       return fail(GTS_ERR_INVALID_GRAPH, "graph offsets decrease at graph " + std::to_string(k));
-  if (row_ptr[0] != 0 || row_ptr[n] != m) return fail(GTS_ERR_INVALID_GRAPH, "row_ptr[0] != 0 or row_ptr[n] != n_edges");
-  uint32_t row_nodes = 0, row_ctas = 0, cross = 0, class_mask = 0;
+  if (ends[0] != 0 || last != m) return fail(GTS_ERR_INVALID_GRAPH, "row_ptr[0] != 0 or row_ptr[n] != n_edges");
+  uint32_t row_nodes = 0, row_ctas = 0;
   for (uint64_t k = 0; k < G; k++) {
-    const uint32_t n0 = noff[k], n1 = noff[k + 1], c0 = coff[k], c1 = coff[k + 1];
-    row_nodes = std::max(row_nodes, n1 - n0);
-    row_ctas = std::max(row_ctas, c1 - c0);
-    for (uint32_t v = n0; v < n1; v++) {
-      if (row_ptr[v + 1] < row_ptr[v]) return fail(GTS_ERR_INVALID_GRAPH, "row_ptr decreases at node " + std::to_string(v));
-      if (ty[v] > GTS_DSMEM) return fail(GTS_ERR_INVALID_GRAPH, "bad type at node " + std::to_string(v));
-      const uint32_t cls_v = (TYPE_CLASS >> (4 * ty[v])) & 15u;
-      if (cls_v < RC_N) class_mask |= 1u << cls_v;
-      if (cls_v == RC_DSM) class_mask |= (1u << RC_LSU) | CM_NOC;
-      if (wp[v] >= W) return fail(GTS_ERR_INVALID_GRAPH, "warp >= warps_per_cta at node " + std::to_string(v));
-      if (cta[v] < c0 || cta[v] >= c1) return fail(GTS_ERR_INVALID_GRAPH, "cta outside its graph at node " + std::to_string(v));
-      if (d->tile && tile[v] != NONE && (ty[v] == GTS_LOAD || ty[v] == GTS_STORE) && tile[v] >= d->n_tiles)
-        return fail(GTS_ERR_INVALID_GRAPH, "tile >= n_tiles at node " + std::to_string(v));
-      for (uint32_t x = row_ptr[v]; x < row_ptr[v + 1]; x++) {
-        if (col[x] <= v || col[x] >= n1)
-          return fail(GTS_ERR_INVALID_GRAPH, "edge " + std::to_string(x) + " must go forward inside its graph");
-        if (ek[x] > 1) return fail(GTS_ERR_INVALID_GRAPH, "bad edge kind at edge " + std::to_string(x));
-        if (cta[col[x]] != cta[v]) cross = 1;
-      }
-    }
-    for (uint32_t c = c0 + 1; c < c1; c++)
-      if (kern[c] < kern[c - 1]) return fail(GTS_ERR_INVALID_GRAPH, "cta_kernel decreases at CTA " + std::to_string(c));
+    row_nodes = std::max(row_nodes, noff[k + 1] - noff[k]);
+    row_ctas = std::max(row_ctas, coff[k + 1] - coff[k]);
   }
 
-  // ---- derived arrays
-  std::vector<uint32_t> indeg(n, 0), first(C * W, NONE), nxt(n, NONE), cnt(C, 0);
-  for (uint64_t x = 0; x < m; x++) indeg[col[x]]++;
-  for (uint64_t v = 0; v < n; v++)
-    if (indeg[v] > MAX_INDEG)
-      return fail(GTS_ERR_UNSUPPORTED, "node " + std::to_string(v) + " has more than 2^24-1 predecessors");
-  for (uint64_t v = n; v-- > 0;) {
-    const uint64_t key = (uint64_t)cta[v] * W + wp[v];
-    nxt[v] = first[key];
-    first[key] = (uint32_t)v;
-  }
-  for (uint64_t v = 0; v < n; v++) cnt[cta[v]]++;
-  std::vector<uint4> rec(n), rng(n);
-  for (uint64_t v = 0; v < n; v++) {
-    rec[v] = make_uint4(work[v], lx[v], nxt[v], (uint32_t)ty[v] | (indeg[v] << 4));
-    const bool tiled = d->tile && tile[v] != NONE && (ty[v] == GTS_LOAD || ty[v] == GTS_STORE);
-    rng[v] = make_uint4(tiled ? tile[v] + 1u : 0u, 0u, row_ptr[v], row_ptr[v + 1]);
-  }
-  std::vector<uint2> succ(m);
-  for (uint64_t x = 0; x < m; x++)
-    succ[x] = make_uint2(col[x], (uint32_t)ek[x] | ((uint32_t)wp[col[x]] << 1) | (cta[col[x]] << 8));
-
-  char *ws = (char *)d->workspace;
-  e = cudaSuccess;
+  // ---- contract checks on the device (Section 4.1 graph): one status read back
+  GraphIn in;
+  in.row_ptr = d->row_ptr; in.col = d->col; in.cta = d->cta; in.work = d->work; in.lx = d->lat_extra;
+  in.kern = d->cta_kernel; in.tile = d->tile; in.ek = d->ekind; in.ty = d->type; in.wp = d->warp;
+  in.n = (uint32_t)n; in.m = (uint32_t)m; in.C = (uint32_t)C; in.W = (uint32_t)W; in.G = (uint32_t)G;
+  in.n_tiles = d->tile ? d->n_tiles : 0u;
+  uint32_t *stat = (uint32_t *)(ws + wl.stat);
+  uint32_t *chi = (uint32_t *)(ws + wl.chi);
+  uint32_t *first = (uint32_t *)(ws + wl.first);
+  uint32_t *cnt = (uint32_t *)(ws + wl.cnt);
+  uint4 *rec = (uint4 *)(ws + wl.rec);
+  uint4 *rng = (uint4 *)(ws + wl.rng);
+  const uint32_t *d_noff = (const uint32_t *)(ws + wl.noff), *d_coff = (const uint32_t *)(ws + wl.coff);
   auto up = [&](size_t off, const void *src, size_t bytes) {
     if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(ws + off, src, bytes, cudaMemcpyHostToDevice, s);
   };
-  up(wl.rec, rec.data(), n * 16);
-  up(wl.rng, rng.data(), n * 16);
-  up(wl.succ, succ.data(), m * 8);
-  up(wl.first, first.data(), C * W * 4);
-  up(wl.cnt, cnt.data(), C * 4);
+  auto zero = [&](size_t off, int value, size_t bytes) {
+    if (e == cudaSuccess && bytes) e = cudaMemsetAsync(ws + off, value, bytes, s);
+  };
   up(wl.noff, noff.data(), (G + 1) * 4);
   up(wl.coff, coff.data(), (G + 1) * 4);
+  zero(wl.stat, 0xFF, GK_NCHECKS * 4);
+  zero(wl.stat + GK_NCHECKS * 4, 0, (GK_WORDS - GK_NCHECKS) * 4);
+  zero(wl.rng, 0, n * 16);
+  zero(wl.first, 0xFF, C * W * 4);
+  zero(wl.cnt, 0, C * 4);
+  zero(wl.chi, 0, C * 4);
+  int dev = 0, sms = 1;
+  if (e == cudaSuccess) e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const uint32_t grid = (uint32_t)std::max<int>(1, sms * 8);
+  if (e == cudaSuccess && n) {
+    k_graph_check<<<grid, 256, 0, s>>>(in, d_noff, d_coff, stat, rng, first, cnt, chi);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess && (n || C)) {
+    k_graph_check2<<<grid, 256, 0, s>>>(in, d_coff, stat, rng, first, cnt, chi);
+    e = cudaGetLastError();
+  }
+  uint32_t st[GK_WORDS];
+  if (e == cudaSuccess) e = cudaMemcpyAsync(st, stat, sizeof(st), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-  if (e != cudaSuccess) return cuda_fail(e, "graph_create: copy to device");
+  if (e != cudaSuccess) return cuda_fail(e, "graph_create: device checks");
+  static const char *what[GK_NCHECKS] = {"row_ptr decreases or exceeds n_edges at node ", "bad type at node ",
+                                         "warp >= warps_per_cta at node ", "cta outside its graph at node ",
+                                         "tile >= n_tiles at node ",
+                                         "edge must go forward inside its graph: edge ",
+                                         "bad edge kind at edge ", "cta_kernel decreases at CTA ",
+                                         "more than 2^24-1 predecessors at node "};
+  for (uint32_t k = 0; k < GK_NCHECKS; k++)
+    if (st[k] != NONE)
+      return fail(k == GK_INDEG ? GTS_ERR_UNSUPPORTED : GTS_ERR_INVALID_GRAPH, what[k] + std::to_string(st[k]));
 
-  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, cross, class_mask,
-                     d->tile ? d->n_tiles : 0u, out);
+  // ---- packing and stream links on the device
+  if (n) {
+    k_graph_pack<<<grid, 256, 0, s>>>(in, rec, rng, (uint2 *)(ws + wl.succ));
+    e = cudaGetLastError();
+  }
+  const uint64_t span = (uint64_t)st[GK_SPAN_LO] | (uint64_t)st[GK_SPAN_HI] << 32;
+  if (e == cudaSuccess && n && span <= 32ull * n + (1ull << 22)) {
+    const uint32_t wpb = 8;
+    k_graph_streams<<<(uint32_t)std::min<uint64_t>((C + wpb - 1) / wpb, 65535), wpb * 32, wpb * W * 4, s>>>(
+        in, first, cnt, chi, rec);
+    e = cudaGetLastError();
+  } else if (e == cudaSuccess && n) {
+    // CTAs interleave over long id ranges (rare): link the streams on the
+    // host from the CTA and warp of every node, then patch the packed records
+    std::vector<uint32_t> hc;
+    std::vector<uint16_t> hw;
+    std::vector<uint4> hrec;
+    e = d2h(hc, d->cta, n, s);
+    if (e == cudaSuccess) e = d2h(hw, d->warp, n, s);
+    if (e == cudaSuccess) e = d2h(hrec, (const uint4 *)rec, n, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess) {
+      std::vector<uint32_t> head(C * W, NONE);
+      for (uint64_t v = n; v-- > 0;) {
+        const uint64_t key = (uint64_t)hc[v] * W + hw[v];
+        hrec[v].z = head[key];
+        head[key] = (uint32_t)v;
+      }
+      e = cudaMemcpyAsync(rec, hrec.data(), n * 16, cudaMemcpyHostToDevice, s);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    }
+  }
+  // the check's temporaries back to zero (the workspace past the packed graph reads as zeros)
+  zero(wl.stat, 0, wl.total - wl.stat);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "graph_create: packing");
+  return make_handle(wl, ws, n, m, C, W, G, noff, coff, d->cta_kernel, row_nodes, row_ctas, st[GK_CROSS] ? 1u : 0u,
+                     st[GK_CLASS], d->tile ? d->n_tiles : 0u, out);
 }
 
 size_t gts_template_workspace_bytes(uint32_t n_templates, uint32_t n_tpl_nodes, uint32_t n_nodes, uint32_t n_edges,
@@ -1443,6 +1640,7 @@ gts_status gts_graph_create_templated(const gts_template_desc *d, void *stream, 
     return fail(GTS_ERR_INVALID_ARG, "null template array");
   if (G > 1 && !d->graph_cta_off) return fail(GTS_ERR_INVALID_ARG, "stacked set needs graph_cta_off");
   if (!d->workspace) return fail(GTS_ERR_INVALID_ARG, "null workspace");
+  if ((uintptr_t)d->workspace % 16 != 0) return fail(GTS_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
   if (d->workspace_bytes < xl.total)
     return fail(GTS_ERR_NOMEM, "workspace too small: need " + std::to_string(xl.total) + " bytes");
   cudaStream_t s = (cudaStream_t)stream;

@@ -433,7 +433,10 @@ def simulate(dgraph: DeviceGraph, dparams: DeviceParams, first_point=0, n_points
 
 
 def utilisation(busy, makespan, params):
-    """Per-class utilisation of each point from its busy server-cycles:
+    """Reporting only: the engine's output is the busy server-cycles per class
+    (GTS_WANT_BUSY, computed in libgts); this turns them into the ratio the
+    paper reports (Section 7.1) for tables and plots, after the simulation.
+    Per-class utilisation of each point from its busy server-cycles:
     busy_r / (servers_r * makespan), servers_r = cap_r * num_sms for the per-SM
     classes, cap_hbm for HBM and cap_noc * ceil(num_sms / cluster_sms) for the
     NoC; 0 where the makespan is 0 or the row has no NoC.  The two L2 entries
