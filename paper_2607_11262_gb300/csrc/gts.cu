@@ -325,6 +325,29 @@ __device__ __forceinline__ void node_cost(const uint32_t *sp, uint32_t type, uin
   lat = (uint64_t)base + lx + max(max(occ, hocc), nocc);
 }
 
+// Dependency counters are read, released into and reset under an L2
+// evict_last policy: a design point's live counters (the nodes near its warp
+// heads) are re-touched soon after their first release, while the trace,
+// written once and never read back, goes out as streaming stores.
+__device__ __forceinline__ uint64_t keep_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ uint2 ld_counters_keep(const uint2 *p, uint64_t pol) {
+  uint2 r;
+  asm volatile("ld.relaxed.gpu.global.L2::cache_hint.v2.u32 {%0, %1}, [%2], %3;"
+               : "=r"(r.x), "=r"(r.y) : "l"(p), "l"(pol) : "memory");
+  return r;
+}
+__device__ __forceinline__ void red_keep(uint2 *c, uint32_t r, uint64_t pol) {  // one released predecessor at r
+  asm volatile("red.relaxed.gpu.global.add.L2::cache_hint.u32 [%0], 1, %1;" ::"l"(&c->x), "l"(pol) : "memory");
+  asm volatile("red.relaxed.gpu.global.max.L2::cache_hint.u32 [%0], %1, %2;" ::"l"(&c->y), "r"(r), "l"(pol) : "memory");
+}
+__device__ __forceinline__ void st_counters_zero_keep(uint2 *p, uint64_t pol) {
+  asm volatile("st.relaxed.gpu.global.L2::cache_hint.v2.u32 [%0], {%1, %1}, %2;" ::"l"(p), "r"(0u), "l"(pol) : "memory");
+}
+
 // Key of slot i computed at cycle t (>= t; INF if it cannot issue yet).
 template <bool EXT>
 __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t sm, uint32_t t) {
@@ -896,6 +919,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       const uint32_t cls = meta & 7u;
       // one round of independent loads: the issued node's record, the next
       // head's record, range and counters, and the successor entries
+      const uint64_t pol = keep_policy();
       const uint4 rv = g.rec[v];
       const uint32_t tkey = l2on ? g.rng[v].x : 0u;  // tile + 1 of the node (0: none)
       uint4 rn = make_uint4(0, 0, 0, 0), qn = rn;
@@ -903,7 +927,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       if (nx != NONE) {
         rn = g.rec[nx];
         qn = g.rng[nx];
-        if (lane == 0) cn = ld_counters(P.scr + (nx - P.n0));
+        if (lane == 0) cn = ld_counters_keep(P.scr + (nx - P.n0), pol);
       }
       uint32_t deg = (meta >> 3) & 31u;
       if (deg == DEG_BIG) deg = g.rng[v].w - sb;
@@ -966,8 +990,8 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       }
       if (lane == 0) {
         if (P.st) {
-          P.st[v - P.n0] = (int32_t)t;
-          P.fi[v - P.n0] = (int32_t)f;
+          __stcs(P.st + (v - P.n0), (int32_t)t);
+          __stcs(P.fi + (v - P.n0), (int32_t)f);
         }
         if (want_digest) digest += mix64(((uint64_t)(v - P.n0) << 32 | t) ^ ((uint64_t)f * 0x9E3779B97F4A7C15ull));
       }
@@ -1033,13 +1057,12 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
           const uint32_t r = __shfl_sync(FULL, rel, j);
           if (lane == 0) {
             uint2 *c = P.scr + (w - P.n0);
-            atomicAdd(&c->x, 1u);
-            atomicMax(&c->y, r);
+            red_keep(c, r, pol);
           }
         }
       }
       __syncwarp();
-      if (lane == 0 && (cn.x | cn.y)) st_counters_zero(P.scr + (nx - P.n0));  // read once: leave the row clean
+      if (lane == 0 && (cn.x | cn.y)) st_counters_zero_keep(P.scr + (nx - P.n0), pol);  // read once: leave the row clean
       cn.x = __shfl_sync(FULL, cn.x, 0);  // the next head's counters (its scratch row is not released into above)
       cn.y = __shfl_sync(FULL, cn.y, 0);
       set_head(P, i, nx, rn, qn, cn, adj_cnt, adj_rdy);

@@ -776,7 +776,7 @@ class Workload:
     params: np.ndarray
 
 
-TEMPLATED = ("gemm512", "wsgemm8192", "wsgemm_small", "fa_fwd", "decoder")
+TEMPLATED = ("gemm512", "wsgemm8192", "wsgemm_small", "fa_fwd", "fa_small", "decoder", "decoder_small")
 
 
 def workload(name: str, points: int | None = None, instances: int | None = None,
@@ -806,6 +806,14 @@ def workload(name: str, points: int | None = None, instances: int | None = None,
         g = fa_fwd(templated=templated)
         p = sweep_params(SEED0 + 3, 1024, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE, AX_ALU_RATE], 1)
         d = "FlashAttention fwd B4 H32 S4096 d128 fp16, non-causal; 1024 points"
+    elif name == "fa_small":
+        g = fa_fwd(batch=1, heads=16, seq=2048, templated=templated)
+        p = sweep_params(SEED0 + 3, 1024, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE, AX_ALU_RATE], 1)
+        d = "FlashAttention fwd B1 H16 S2048 d128 (profiling-size case of the fa_fwd shape); 1024 points"
+    elif name == "decoder_small":
+        g = decoder_layer(hidden=1024, heads=8, ffn=2816, tokens=2048, seq=512, templated=templated)
+        p = sweep_params(SEED0 + 4, 512, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE, AX_ALU_RATE], 1)
+        d = "decoder layer hidden 1024, 8 heads, FFN 2816, 4x512 tokens (profiling-size case of the decoder shape); 512 points"
     elif name == "decoder":
         g = decoder_layer(templated=templated)
         p = sweep_params(SEED0 + 4, 512, [AX_SMS, AX_HBM, AX_TMA_LAT, AX_MMA_RATE, AX_ALU_RATE], 1)

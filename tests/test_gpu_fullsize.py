@@ -57,7 +57,7 @@ def test_axis_sample_covers_both_ends_and_middle():
         assert vals.min() == p[:, k].min() and vals.max() == p[:, k].max()
 
 
-@pytest.mark.parametrize("name", ["gemm512", "wsgemm8192", "fa_fwd", "decoder", "stress"])
+@pytest.mark.parametrize("name", list(W.WORKLOADS))
 def test_full_size_workload_every_point(gts_mod, name):
     import torch
     gts = gts_mod

@@ -69,3 +69,52 @@ def test_malformed_template_sets_are_refused(gts_mod):
         with pytest.raises(gts.GtsError) as e:
             gts.DeviceGraph(_broken(ts, **case))
         assert e.value.status == gts.GTS_ERR_INVALID_GRAPH, case.keys()
+
+
+def _random_template(rng, warps, n, fan=False):
+    t = W.CtaTemplate(warps)
+    for v in range(n):
+        t.node(int(rng.integers(0, 7)), int(rng.integers(0, warps)), work=int(rng.integers(0, 9)),
+               lat_extra=int(rng.integers(0, 3)))
+    for v in range(1, n):
+        for u in rng.choice(v, size=min(v, int(rng.integers(0, 3))), replace=False):
+            t.edge(int(u), v, int(rng.integers(0, 2)))
+    if fan and n > 40:  # node 0 feeds every later node: more than 32 successors
+        have = set(zip(t.es, t.ed))
+        for v in range(1, n):
+            if (0, v) not in have:
+                t.edge(0, v, W.DATA)
+    return t
+
+
+def test_random_template_sets(gts_mod):
+    """Random template sets (several templates, one unused, a node with more than
+    32 successors, stacked graphs, kernel gates), expanded on the device and
+    simulated: bit-exact against the oracle on the expanded logical graph."""
+    import torch
+
+    from oracle import run as oracle_run
+    from tests import gpu_helpers as H
+    from tests import tinygraphs as TG
+    gts = gts_mod
+    rng = np.random.default_rng(31)
+    for case in range(6):
+        warps = int(rng.integers(1, 5))
+        tpls = [_random_template(rng, warps, int(rng.integers(1, 60)), fan=(k == 0)) for k in range(4)]
+        C = int(rng.integers(2, 14))
+        ct = rng.integers(0, 3, C)          # template 3 is never used
+        kern = np.sort(rng.integers(0, 3, C)) if case % 2 else np.zeros(C, np.int64)
+        goff = None
+        if case >= 3:                       # two stacked graphs
+            cut = int(rng.integers(1, C))
+            goff = [0, cut, C]
+            kern = np.concatenate([np.sort(kern[:cut]), np.sort(kern[cut:])])
+        ts = W.template_set(f"rand{case}", warps, tpls, ct, kern, goff)
+        g = ts.expand()
+        prms = np.stack([TG.small_params(rng) for _ in range(8)])
+        if goff is not None:
+            prms[:, W.P_GRAPH_INDEX] = np.arange(8) % 2
+        res = H.run_gpu(ts, prms)
+        torch.cuda.synchronize()
+        for q in range(prms.shape[0]):
+            H.assert_point_equal(g, prms[q], res, q, oracle_run.simulate(g, prms[q]))

@@ -63,7 +63,8 @@ SIZES = {"gemm512": (2176, 4736, 64), "wsgemm8192": (1581056, 1842144, 4096), "f
 
 
 def test_every_named_workload_keeps_the_contract():
-    for name in ("gemm512", "wsgemm_small", "wsgemm8192", "fa_fwd", "decoder", "pipelines", "noc_fusion", "l2_gemm"):
+    for name in ("gemm512", "wsgemm_small", "wsgemm8192", "fa_fwd", "fa_small", "decoder", "decoder_small",
+                 "pipelines", "noc_fusion", "l2_gemm"):
         w = W.workload(name)
         _contract(w.graph)
         assert w.params.shape[1] == W.NPARAM and w.params.dtype == np.int32, name
