@@ -480,14 +480,15 @@ def main():
         torch.distributed.destroy_process_group()
 
 
-def measure_e2e(graph, params, gts, stream, reps=2, templates=None, chunk_bytes=1 << 30):
+def measure_e2e(graph, params, gts, stream, reps=2, templates=None, chunk_bytes=1 << 30, copy_streams=4):
     """Same metric through the public API from pinned host buffers, every step:
     graph and parameter upload (host->device), graph packing, the batch, and
     the device->host read of the whole result -- the start/finish trace of
     every point, then the makespans and statuses.  The trace crosses the link
-    in chunks of rows into two reused pinned buffers of ``chunk_bytes`` (a
-    consumer would write each chunk out or reduce it as it arrives; 52 GB of
-    trace per wsgemm8192 step is not kept in host memory).  With ``templates``
+    in chunks of rows, spread over ``copy_streams`` streams that each reuse one
+    pinned buffer of ``chunk_bytes`` (a consumer would write each chunk out or
+    reduce it as it arrives; 52 GB of trace per wsgemm8192 step is not kept in
+    host memory).  With ``templates``
     (the same graph as a TemplateSet) the graph goes in template-shared form:
     templates and the CTA table are uploaded and libgts expands them."""
     import torch
@@ -504,7 +505,8 @@ def measure_e2e(graph, params, gts, stream, reps=2, templates=None, chunk_bytes=
     hp = torch.from_numpy(np.ascontiguousarray(params, np.int32).reshape(-1)).pin_memory()
     h_mk = torch.empty(P, dtype=torch.int32).pin_memory()
     h_st = torch.empty(P, dtype=torch.int32).pin_memory()
-    ring = [torch.empty(chunk_bytes // 4, dtype=torch.int32).pin_memory() for _ in range(2)]
+    ring = [torch.empty(chunk_bytes // 4, dtype=torch.int32).pin_memory() for _ in range(copy_streams)]
+    copiers = [torch.cuda.Stream() for _ in range(copy_streams)]
     # inputs, plus the processing order libgts uploads (4 B per point, gts_params_set_order)
     h2d = sum(t.numel() * t.element_size() for t in host.values()) + hp.numel() * 4 + 4 * P
     flags = gts.GTS_FULL_TRACE | gts.GTS_SCRATCH_CLEAN
@@ -521,14 +523,21 @@ def measure_e2e(graph, params, gts, stream, reps=2, templates=None, chunk_bytes=
             out = gts.alloc_outputs(dg, P, flags)
             scratch = gts.alloc_scratch(dg, dpp, flags, stream=stream)
             gts.simulate(dg, dpp, flags=flags, out=out, scratch=scratch, stream=stream)
+            done = torch.cuda.Event()
+            done.record(stream)
             rows = max(1, (chunk_bytes // 4) // max(dg.row_nodes, 1))
             d2h, k = 0, 0
+            for cs in copiers:
+                cs.wait_event(done)
             for trace in (out.start, out.finish):
                 for r0 in range(0, P, rows):
                     part = trace[r0:r0 + rows].reshape(-1)
-                    ring[k][:part.numel()].copy_(part, non_blocking=True)
+                    with torch.cuda.stream(copiers[k]):
+                        ring[k][:part.numel()].copy_(part, non_blocking=True)
                     d2h += part.numel() * 4
-                    k ^= 1
+                    k = (k + 1) % copy_streams
+            for cs in copiers:
+                stream.wait_stream(cs)
             h_mk.copy_(out.makespan, non_blocking=True)
             h_st.copy_(out.status, non_blocking=True)
             d2h += 8 * P
@@ -539,8 +548,8 @@ def measure_e2e(graph, params, gts, stream, reps=2, templates=None, chunk_bytes=
     t = min(times)
     return {"value": node_points / t, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "seconds_per_step": t, "graph_input": "template-shared" if templates is not None else "logical",
-            "trace_to_host": f"start and finish rows in {2 * ((P + rows - 1) // rows)} chunks into two "
-                             f"{chunk_bytes >> 20} MiB pinned buffers"}
+            "trace_to_host": f"start and finish rows in {2 * ((P + rows - 1) // rows)} chunks over {copy_streams} "
+                             f"copy streams, each into its own {chunk_bytes >> 20} MiB pinned buffer"}
 
 
 if __name__ == "__main__":

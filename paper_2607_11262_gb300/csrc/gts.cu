@@ -529,6 +529,52 @@ __device__ __forceinline__ void refresh_sm(const Pt &P, uint32_t s, uint32_t t, 
   __syncwarp();
 }
 
+// Warp-parallel, SMs of at most 16 slots and at most 512 SMs: SM s's record
+// (as refresh_sm) and the owner lane's best (as refresh_owner after it) in
+// one pass.  Lanes below per key SM s's slots; lane 16 + j reads the record of
+// the owner's j-th SM (owner + 32 j) unless it is s; the two minima are
+// independent reductions over the same values.
+template <bool EXT>
+__device__ __forceinline__ void refresh_sm_owner(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane, uint64_t &b,
+                                                 uint32_t &bsl) {
+  const uint32_t per = P.L.per, i0 = s * per, owner = s & 31u, l = (uint32_t)lane;
+  uint64_t vs = INF64, vo = INF64;
+  uint32_t hk = INF, so = 0;
+  if (l < per && i0 + l < P.L.S) {
+    const uint32_t k = slot_key<EXT>(P, i0 + l, s, t);
+    if (k != INF) {
+      const uint32_t h = P.slot(i0 + l)[F_HID];
+      const bool hb = (h & HBM_BIT) != 0u;
+      vs = pack(hb ? max(k, H) : k, h & ID_MASK);
+      if (hb) hk = k;
+    }
+  } else if (l >= 16u) {
+    const uint32_t sj = owner + 32u * (l - 16u);
+    if (sj < P.L.NS && sj != s) {
+      const uint2 o = *reinterpret_cast<const uint2 *>(P.smrec(sj));
+      vo = pack(o.y, o.x);
+      so = P.smrec(sj)[2];
+    }
+  }
+  uint32_t wa, wb;
+  const uint64_t ma = warp_min64(vs, wa);
+  const uint64_t mb = warp_min64(vs < vo ? vs : vo, wb);
+  const uint32_t hmin = __reduce_min_sync(FULL, hk);
+  const uint32_t sb = __shfl_sync(FULL, l < 16u ? i0 + l : so, wb);
+  if (lane == 0) {
+    uint32_t *o = P.smrec(s);
+    o[0] = (uint32_t)ma;
+    o[1] = (uint32_t)(ma >> 32);
+    o[2] = ma == INF64 ? 0u : i0 + wa;
+    o[3] = hmin;
+  }
+  if (l == owner) {
+    b = mb;
+    bsl = mb == INF64 ? 0u : sb;
+  }
+  __syncwarp();
+}
+
 // One lane: recompute the record of SM s at cycle t and horizon H.
 template <bool EXT>
 __device__ __forceinline__ void rescan_sm_lane(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
@@ -1102,6 +1148,17 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane<EXT>(P, s, t, C.H);
         __syncwarp();
         b = lane_best(P, lane, bsl);
+      } else if (C.H == prevH && P.L.per <= 16u && P.L.NS <= 512u && !(EXT && P.L.nsub)) {
+        refresh_sm_owner<EXT>(P, sm, t, C.H, lane, b, bsl);
+        if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
+          const uint32_t g0 = div16(sm, P.mCsms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
+          for (uint32_t s = g0 + lane; s < g1; s += 32)
+            if (s != sm) rescan_sm_lane<EXT>(P, s, t, C.H);
+          __syncwarp();
+          bool mine = false;
+          for (uint32_t s = g0; s < g1; s++) mine |= s != sm && (s & 31u) == (uint32_t)lane;
+          if (mine) b = lane_best(P, lane, bsl);
+        }
       } else {
         refresh_sm<EXT>(P, sm, t, C.H, lane);
         if (C.H != prevH && P.L.per >= 8u && !(EXT && P.L.nsub)) {
@@ -1875,9 +1932,9 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
     }
   }
   uint64_t warps = (uint64_t)std::max(best_w, 1u) * sms;
-  // a batch smaller than one wave: blocks small enough that every SM gets one
-  // before any gets two (the block scheduler fills SMs breadth first)
-  if (np < warps) pl.wpb = std::max(1u, std::min(pl.wpb, np / (uint32_t)sms));
+  // a batch smaller than one wave: one design point per block, so that the
+  // block scheduler (which fills SMs breadth first) spreads the points evenly
+  if (np < warps) pl.wpb = 1u;
   warps = std::min<uint64_t>(warps, np);
   if (limit_by_scratch) {
     const uint64_t row = scratch_row_bytes(g);
