@@ -3,8 +3,8 @@
  *
  * TEST INFRASTRUCTURE ONLY.  This file is the CPU oracle that the CUDA path is
  * checked against.  Only the tests, the smoke check and the benchmark's CPU
- * baseline may load it; the product path never does.  It shares no code,
- * header or table with the CUDA library.
+ * baseline and reference arm may load it; the product path never does.  It
+ * shares no code, header or table with the CUDA library.
  *
  * What it computes (graph-driven simulation backend, Section 5):
  *   Given a tile graph G = (V, E) (Section 4.1) and one hardware parameter row,

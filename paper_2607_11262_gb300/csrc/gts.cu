@@ -23,7 +23,8 @@
 //    minimum over its heads; lane l owns SMs l, l+32, ... and keeps the
 //    minimum over them in registers; the warp takes the minimum over lanes
 //    with two __reduce_min_sync.  After an issue the issuing SM's keys and
-//    summary are recomputed warp-parallel, then its owner lane's minimum;
+//    summary are recomputed warp-parallel together with its owner lane's
+//    minimum (one pass, two independent reductions, for SMs of <= 16 slots);
 //    when H moves, the SMs whose HBM heads it overtakes are recomputed (each
 //    lane its own SMs, or one SM at a time a slot per lane when SMs hold 8
 //    slots or more).  A release into a head of another CTA recomputes every
