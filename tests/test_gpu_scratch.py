@@ -80,9 +80,12 @@ def test_clean_scratch_reused_with_error_points(gts):
         if first is None:
             first = res
             _check(w.graph, p, res)
-        else:
-            for k in ("status", "makespan", "start", "finish", "digest"):
+        else:  # a failed point's trace rows are unspecified (the ABI says so): compare the OK points' rows
+            ok = first["status"] == 0
+            for k in ("status", "makespan", "digest"):
                 assert np.array_equal(res[k], first[k]), k
+            for k in ("start", "finish"):
+                assert np.array_equal(res[k][ok], first[k][ok]), k
 
 
 def test_dirty_scratch_without_flag_is_cleared(gts):
