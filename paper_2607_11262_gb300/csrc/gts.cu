@@ -143,8 +143,11 @@ constexpr uint32_t O_BASE = GTS_NPARAM + 14; // 8 words: base latency per node t
 constexpr uint32_t O_L2B = O_BASE + 8;
 constexpr uint32_t O_DYN = GTS_NPARAM + 24;  // first per-point array
 static_assert(O_MAG % 2 == 0, "division constants are 8-byte words");
-// slot record (5 words): id|HBM, rdy, pending<<8 | deg<<3 | class, next, successor begin
-constexpr uint32_t F_HID = 0, F_RDY = 1, F_META = 2, F_NXT = 3, F_SB = 4, SLOT_WORDS = 5;
+// slot record (4 words, one 16-byte vector): id|HBM, rdy, pending<<8 | deg<<3 | class, next node of the stream.
+// The successor-list start is read from the node's range record when it issues, which keeps a point at 4 words
+// per warp slot (at 132 SMs x 3 warps, 8 two-warp blocks fit on an SM instead of 7).
+constexpr uint32_t F_HID = 0, F_RDY = 1, F_META = 2, F_NXT = 3, SLOT_WORDS = 4;
+static_assert(O_DYN % 4 == 0 && SLOT_WORDS == 4 && F_NXT == 3, "warp slots are read and written as 16-byte vectors");
 // SM record (4 words): best id, best effective cycle, best slot, min key of its HBM heads
 constexpr uint32_t SM_WORDS = 4;
 static_assert(SM_WORDS % 2 == 0, "SM records are read as 8-byte pairs");
@@ -352,11 +355,11 @@ __device__ __forceinline__ void st_counters_zero_keep(uint2 *p, uint64_t pol) {
 // Key of slot i computed at cycle t (>= t; INF if it cannot issue yet).
 template <bool EXT>
 __device__ __forceinline__ uint32_t slot_key(const Pt &P, uint32_t i, uint32_t sm, uint32_t t) {
-  const uint32_t *sl = P.slot(i);
-  const uint32_t h = sl[F_HID];
-  const uint32_t meta = sl[F_META];
+  const uint4 e = *reinterpret_cast<const uint4 *>(P.slot(i));  // {id|HBM, rdy, meta, next}
+  const uint32_t h = e.x;
+  const uint32_t meta = e.z;
   if (h == NONE || (meta >> 8) != 0u) return INF;
-  uint32_t k = max(sl[F_RDY], t);
+  uint32_t k = max(e.y, t);
   const uint32_t cls = meta & 7u;
   if (cls != RC_NONE) {
     const uint32_t sc = EXT && cls == RC_DSM ? RC_LSU : cls;
@@ -648,11 +651,8 @@ __device__ __forceinline__ void set_head(const Pt &P, uint32_t i, uint32_t v, ui
   const uint32_t type = r.w & 15u;
   const uint32_t pend = (r.w >> 4) - c.x - adj_cnt;
   const uint32_t deg = min(q.w - q.z, DEG_BIG);
-  sl[F_HID] = v | (((TYPE_HBM >> type) & 1u) ? HBM_BIT : 0u);
-  sl[F_RDY] = max(c.y, adj_rdy);
-  sl[F_META] = ((TYPE_CLASS >> (4 * type)) & 15u) | (deg << 3) | (pend << 8);
-  sl[F_NXT] = r.z;
-  sl[F_SB] = q.z;
+  *reinterpret_cast<uint4 *>(sl) = make_uint4(v | (((TYPE_HBM >> type) & 1u) ? HBM_BIT : 0u), max(c.y, adj_rdy),
+                                              ((TYPE_CLASS >> (4 * type)) & 15u) | (deg << 3) | (pend << 8), r.z);
 }
 
 struct Clock {
@@ -962,13 +962,16 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       const uint32_t cs = div16(i, P.mW);
       const uint32_t sm = div16(cs, P.mCps);
       const uint32_t *sl = P.slot(i);
-      const uint32_t hidv = sl[F_HID], meta = sl[F_META], nx = sl[F_NXT], sb = sl[F_SB];
+      const uint4 se = *reinterpret_cast<const uint4 *>(sl);
+      const uint32_t hidv = se.x, meta = se.z, nx = se.w;
       const uint32_t cls = meta & 7u;
-      // one round of independent loads: the issued node's record, the next
-      // head's record, range and counters, and the successor entries
+      // one round of loads: the issued node's record and range (its successor-list
+      // start), the next head's record, range and counters; then the successor entries
       const uint64_t pol = keep_policy();
       const uint4 rv = g.rec[v];
-      const uint32_t tkey = l2on ? g.rng[v].x : 0u;  // tile + 1 of the node (0: none)
+      const uint4 qv = g.rng[v];
+      const uint32_t tkey = l2on ? qv.x : 0u;  // tile + 1 of the node (0: none)
+      const uint32_t sb = qv.z;
       uint4 rn = make_uint4(0, 0, 0, 0), qn = rn;
       uint2 cn = make_uint2(0, 0);
       if (nx != NONE) {
@@ -977,7 +980,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         if (lane == 0) cn = ld_counters_keep(P.scr + (nx - P.n0), pol);
       }
       uint32_t deg = (meta >> 3) & 31u;
-      if (deg == DEG_BIG) deg = g.rng[v].w - sb;
+      if (deg == DEG_BIG) deg = qv.w - sb;
       uint2 ew = make_uint2(NONE, 0);
       if ((uint32_t)lane < deg) ew = g.succ[sb + lane];
       uint32_t occ, hocc, nocc;

@@ -66,7 +66,7 @@ def test_many_cta_slots_per_sm():
 
 
 def test_row_too_large_for_one_warp_is_unsupported():
-    # 6,000 SMs x 1 CTA slot with 6,000 one-node CTAs: about 48 bytes of
+    # 6,000 SMs x 1 CTA slot with 6,000 one-node CTAs: about 44 bytes of
     # on-chip state per SM, more than one warp may keep in shared memory; the
     # other rows still run
     n = 6000
