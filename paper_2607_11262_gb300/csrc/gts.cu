@@ -786,7 +786,8 @@ __device__ __forceinline__ uint32_t first_point_of(const uint32_t *order, uint32
 // from one SM sub-partition's 16K-register file, allocated 8 per thread at a
 // time: 4 warps fit per sub-partition up to 128 registers, 3 up to 168, 2
 // above.  The plain instance is held to 128 (16 warps per SM; shared memory
-// allows 14 on the large rows), the extended one to 168 (12 warps per SM).
+// also allows 16 on rows of 132 SMs x 3 warps), the extended one to 168 (12
+// warps per SM).
 template <bool EXT>
 __global__ void __launch_bounds__(MAX_WPB * 32, EXT ? 3 : 4)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
