@@ -27,8 +27,11 @@
 //    minimum (one pass, two independent reductions, for SMs of <= 16 slots);
 //    when H moves, the SMs whose HBM heads it overtakes are recomputed (each
 //    lane its own SMs, or one SM at a time a slot per lane when SMs hold 8
-//    slots or more).  A release into a head of another CTA recomputes every
-//    SM (the extended instance: the SMs it reached).
+//    slots or more).  When every SM has fewer than 8 slots, an SM whose only
+//    issuable HBM head is one keeps that head apart in its summary and takes
+//    its effective cycle max(key, H) when the summary is read, so such SMs
+//    need no recomputation when H moves.  A release into a head of another
+//    CTA recomputes every SM (the extended instance: the SMs it reached).
 //  * The issue itself runs in every lane on broadcast values (no divergence);
 //    only global atomics and scratch-counter reads are lane 0's.
 //  * Dependency release (Section 5.1).  An issued node releases each
@@ -295,7 +298,7 @@ struct Pt {
   uint32_t caps;     // 6 bits per class: servers of class r (0: class unused)
   uint32_t policy;   // GTS_POLICY_*; L.nsub > 0 for the per-subpartition policies
   uint32_t mW, mCps; // div16 constants of W and ctas_per_sm; slot and CTA-slot indices stay below
-                     // 2^16 because 5-word slot records of a point fit in MAX_SMEM_BYTES
+                     // 2^16 because the 4-word slot records of a point fit in MAX_SMEM_BYTES
   uint32_t mSub, mCsms;  // div16 constants of the scheduler count and the SMs per NoC group
   __device__ __forceinline__ uint32_t cls_off(uint32_t r) const { return (uint32_t)(offs >> (8 * r)) & 255u; }
   __device__ __forceinline__ uint32_t cls_cap(uint32_t r) const { return (caps >> (6 * r)) & 63u; }
@@ -637,6 +640,193 @@ __device__ __forceinline__ void refresh_owner(const Pt &P, uint32_t owner, int l
   if ((uint32_t)lane == owner) { b = best; bsl = slot; }
 }
 
+// ---- split SM records (plain instance, SMs of fewer than 8 slots).  An SM
+// with exactly one issuable HBM head keeps it apart from its other heads:
+// words 0-1 hold the best NON-HBM head (effective cycle, id), word 2 that
+// head's slot | the HBM head's slot << 16, word 3 the HBM head's key.  The HBM
+// head's effective cycle max(key, H) is taken where the record is read, so a
+// horizon move needs no rescan of such an SM.  Any other SM keeps the whole
+// record (best head at the horizon of its last refresh, slot | SPLIT_NONE,
+// least HBM key) and is rescanned when H passes that key.
+constexpr uint32_t SPLIT_NONE = 0xFFFF0000u;
+
+__device__ __forceinline__ void put_split_rec(const Pt &P, uint32_t s, uint64_t nh, uint32_t nhslot, uint64_t all,
+                                              uint32_t allslot, uint32_t hcnt, uint32_t hslot, uint32_t hmin) {
+  uint32_t *o = P.smrec(s);
+  const bool one = hcnt == 1u;
+  const uint64_t v = one ? nh : all;
+  o[0] = (uint32_t)v;
+  o[1] = (uint32_t)(v >> 32);
+  o[2] = (v == INF64 ? 0u : (one ? nhslot : allslot)) | (one ? hslot << 16 : SPLIT_NONE);
+  o[3] = hmin;
+}
+
+// Best (effective cycle << 32 | id) of SM s at horizon H, and its slot.
+__device__ __forceinline__ uint64_t split_sm_best(const Pt &P, uint32_t s, uint32_t H, uint32_t &slot) {
+  const uint32_t *o = P.smrec(s);
+  const uint2 a = *reinterpret_cast<const uint2 *>(o);
+  const uint2 c = *reinterpret_cast<const uint2 *>(o + 2);
+  uint64_t v = pack(a.y, a.x);
+  slot = c.x & 0xFFFFu;
+  if ((c.x >> 16) != 0xFFFFu) {
+    const uint64_t hv = pack(max(c.y, H), P.slot(c.x >> 16)[F_HID] & ID_MASK);
+    if (hv < v) {
+      v = hv;
+      slot = c.x >> 16;
+    }
+  }
+  return v;
+}
+
+// Warp-parallel refresh of SM s (all its slots in one round of lanes).
+__device__ __forceinline__ void split_refresh_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane) {
+  const uint32_t i0 = s * P.L.per, i = i0 + lane;
+  uint64_t val = INF64;
+  uint32_t hk = INF;
+  bool hf = false;
+  if (lane < (int)P.L.per && i < P.L.S) {
+    const uint32_t k = slot_key<false>(P, i, s, t);
+    const uint32_t h = P.slot(i)[F_HID];
+    if (k != INF) {
+      hf = (h & HBM_BIT) != 0u;
+      val = pack(hf ? max(k, H) : k, h & ID_MASK);
+      if (hf) hk = k;
+    }
+  }
+  const uint32_t hcnt = __popc(__ballot_sync(FULL, hf));
+  uint32_t who;
+  const uint64_t m = warp_min64(hcnt == 1u && hf ? INF64 : val, who);
+  const uint32_t hmin = __reduce_min_sync(FULL, hk);
+  if (hcnt == 1u ? hf : lane == 0) put_split_rec(P, s, m, i0 + who, m, i0 + who, hcnt, i, hmin);
+  __syncwarp();
+}
+
+// Warp-parallel, as refresh_sm_owner: SM s's record and the owner lane's best
+// (b, bsl) from two independent reductions over the same values.
+__device__ __forceinline__ void split_refresh_sm_owner(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane,
+                                                       uint64_t &b, uint32_t &bsl) {
+  const uint32_t per = P.L.per, i0 = s * per, owner = s & 31u, l = (uint32_t)lane;
+  uint64_t vs = INF64, vo = INF64;
+  uint32_t hk = INF, so = 0;
+  bool hf = false;
+  if (l < per && i0 + l < P.L.S) {
+    const uint32_t k = slot_key<false>(P, i0 + l, s, t);
+    if (k != INF) {
+      const uint32_t h = P.slot(i0 + l)[F_HID];
+      hf = (h & HBM_BIT) != 0u;
+      vs = pack(hf ? max(k, H) : k, h & ID_MASK);
+      if (hf) hk = k;
+    }
+  } else if (l >= 16u) {
+    const uint32_t sj = owner + 32u * (l - 16u);
+    if (sj < P.L.NS && sj != s) vo = split_sm_best(P, sj, H, so);
+  }
+  const bool one = __popc(__ballot_sync(FULL, hf)) == 1u;
+  uint32_t wa, wb;
+  const uint64_t ma = warp_min64(one && hf ? INF64 : vs, wa);
+  const uint64_t mb = warp_min64(vs < vo ? vs : vo, wb);
+  const uint32_t hmin = __reduce_min_sync(FULL, hk);
+  const uint32_t sb = __shfl_sync(FULL, l < 16u ? i0 + l : so, wb);
+  if (one ? hf : lane == 0) {
+    uint32_t *o = P.smrec(s);
+    o[0] = (uint32_t)ma;
+    o[1] = (uint32_t)(ma >> 32);
+    o[2] = (ma == INF64 ? 0u : i0 + wa) | (one ? (i0 + l) << 16 : SPLIT_NONE);
+    o[3] = hmin;
+  }
+  if (l == owner) {
+    b = mb;
+    bsl = mb == INF64 ? 0u : sb;
+  }
+  __syncwarp();
+}
+
+// One lane: recompute the record of SM s at cycle t and horizon H.
+__device__ __forceinline__ void split_rescan_sm_lane(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
+  const uint32_t i0 = s * P.L.per, i1 = min(i0 + P.L.per, P.L.S);
+  uint64_t best = INF64, nbest = INF64;
+  uint32_t bsl = 0, nsl = 0, hmin = INF, hcnt = 0, hslot = 0;
+  for (uint32_t i = i0; i < i1; i++) {
+    const uint32_t k = slot_key<false>(P, i, s, t);
+    if (k == INF) continue;
+    const uint32_t h = P.slot(i)[F_HID];
+    const bool hb = (h & HBM_BIT) != 0u;
+    const uint64_t val = pack(hb ? max(k, H) : k, h & ID_MASK);
+    if (hb) {
+      hmin = min(hmin, k);
+      hcnt++;
+      hslot = i;
+    } else if (val < nbest) {
+      nbest = val;
+      nsl = i;
+    }
+    if (val < best) { best = val; bsl = i; }
+  }
+  put_split_rec(P, s, nbest, nsl, best, bsl, hcnt, hslot, hmin);
+}
+
+__device__ __forceinline__ uint64_t split_lane_best(const Pt &P, int lane, uint32_t H, uint32_t &slot) {
+  uint64_t b = INF64;
+  slot = 0;
+  for (uint32_t s = lane; s < P.L.NS; s += 32) {
+    uint32_t sl;
+    const uint64_t v = split_sm_best(P, s, H, sl);
+    if (v < b) { b = v; slot = sl; }
+  }
+  return b;
+}
+
+__device__ __forceinline__ void split_refresh_owner(const Pt &P, uint32_t owner, int lane, uint32_t H, uint64_t &b,
+                                                    uint32_t &bsl) {
+  uint64_t best = INF64;
+  uint32_t slot = 0;
+  for (uint32_t base = owner; base < P.L.NS; base += 32 * 32) {
+    const uint32_t s = base + 32u * lane;
+    uint64_t val = INF64;
+    uint32_t sl = 0;
+    if (s < P.L.NS) val = split_sm_best(P, s, H, sl);
+    uint32_t who;
+    const uint64_t m = warp_min64(val, who);
+    const uint32_t ws = __shfl_sync(FULL, sl, who);
+    if (m < best) { best = m; slot = ws; }
+  }
+  if ((uint32_t)lane == owner) { b = best; bsl = slot; }
+}
+
+// Refresh entry points of the kernel: the split forms in the instance that
+// keeps split SM records, the plain ones otherwise.
+template <bool EXT, bool SPL>
+__device__ __forceinline__ void r_sm(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane) {
+  if constexpr (SPL) split_refresh_sm(P, s, t, H, lane); else refresh_sm<EXT>(P, s, t, H, lane);
+}
+template <bool EXT, bool SPL>
+__device__ __forceinline__ void r_sm_owner(const Pt &P, uint32_t s, uint32_t t, uint32_t H, int lane, uint64_t &b,
+                                           uint32_t &bsl) {
+  if constexpr (SPL) split_refresh_sm_owner(P, s, t, H, lane, b, bsl); else refresh_sm_owner<EXT>(P, s, t, H, lane, b, bsl);
+}
+template <bool EXT, bool SPL>
+__device__ __forceinline__ void r_rescan(const Pt &P, uint32_t s, uint32_t t, uint32_t H) {
+  if constexpr (SPL) split_rescan_sm_lane(P, s, t, H); else rescan_sm_lane<EXT>(P, s, t, H);
+}
+template <bool SPL>
+__device__ __forceinline__ uint64_t r_lane_best(const Pt &P, int lane, uint32_t H, uint32_t &slot) {
+  if constexpr (SPL) return split_lane_best(P, lane, H, slot); else return lane_best(P, lane, slot);
+}
+template <bool SPL>
+__device__ __forceinline__ void r_owner(const Pt &P, uint32_t owner, int lane, uint32_t H, uint64_t &b, uint32_t &bsl) {
+  if constexpr (SPL) split_refresh_owner(P, owner, lane, H, b, bsl); else refresh_owner(P, owner, lane, b, bsl);
+}
+// SM s's record must be rescanned once H passes its least HBM key (whole records only).
+template <bool SPL>
+__device__ __forceinline__ bool r_stale(const Pt &P, uint32_t s, uint32_t H) {
+  if constexpr (SPL) {
+    const uint2 c = *reinterpret_cast<const uint2 *>(P.smrec(s) + 2);
+    return c.y < H && (c.x >> 16) == 0xFFFFu;
+  } else {
+    return P.smrec(s)[3] < H;
+  }
+}
+
 // Slot i takes node v as its head (v == NONE: stream exhausted); adj_cnt /
 // adj_rdy are releases the caller applied directly.  Every lane writes the
 // same values.
@@ -665,7 +855,7 @@ struct Clock {
 
 // Retire finished CTAs and launch as many CTAs as fit at cycle t (Section 5.1
 // TB scheduler; kernel-boundary gate).  Returns false on step-limit.
-template <bool EXT>
+template <bool EXT, bool SPL>
 __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_row, int lane, uint64_t &b,
                             uint32_t &bsl) {
   const uint32_t t = C.t;
@@ -723,8 +913,8 @@ __device__ bool launch_ctas(const DevGraph &g, Pt &P, Clock &C, int32_t *cta_sm_
     }
     __syncwarp();
     const uint32_t s = div16(freeslot, P.mCps);
-    refresh_sm<EXT>(P, s, t, C.H, lane);
-    refresh_owner(P, s & 31u, lane, b, bsl);
+    r_sm<EXT, SPL>(P, s, t, C.H, lane);
+    r_owner<SPL>(P, s & 31u, lane, C.H, b, bsl);
     C.next_cta++;
   }
 }
@@ -781,14 +971,17 @@ __device__ __forceinline__ uint32_t first_point_of(const uint32_t *order, uint32
 }
 
 // EXT: the kernel instance that also runs the per-subpartition issue policies
-// and the NoC of DSMEM nodes; the host launches the plain instance when no row
-// asks for a policy and the graph has no DSMEM node.  A warp's registers come
+// and the NoC of DSMEM nodes; the host launches a plain instance when no row
+// asks for a policy and the graph has no DSMEM node.  SPL: the plain instance
+// that keeps split SM records, launched when every row's SMs have fewer than 8
+// warp slots (the record forms are described above split_sm_best); the other
+// plain instance keeps whole records only.  A warp's registers come
 // from one SM sub-partition's 16K-register file, allocated 8 per thread at a
 // time: 4 warps fit per sub-partition up to 128 registers, 3 up to 168, 2
 // above.  The plain instance is held to 128 (16 warps per SM; shared memory
 // also allows 16 on rows of 132 SMs x 3 warps), the extended one to 168 (12
 // warps per SM).
-template <bool EXT>
+template <bool EXT, bool SPL>
 __global__ void __launch_bounds__(MAX_WPB * 32, EXT ? 3 : 4)
 k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point, uint32_t n_points, uint32_t flags,
            int32_t *d_start, int32_t *d_finish, int32_t *d_makespan, int32_t *d_status, uint64_t *d_digest,
@@ -831,7 +1024,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     const bool l2on = EXT && status == GTS_OK && prm[GTS_P_L2_BYTES] != 0;
     if (status == GTS_OK) {
       if (!make_layout(prm, CG, P.W, g.class_mask, P.L) || P.L.words > budget_words ||
-          (!EXT && (P.L.nsub || P.L.cap_noc || prm[GTS_P_L2_BYTES] != 0)))
+          (!EXT && (P.L.nsub || P.L.cap_noc || prm[GTS_P_L2_BYTES] != 0)) || (SPL && P.L.per >= 8u))
         status = GTS_ERR_UNSUPPORTED;
     }
     if (status != GTS_OK) {
@@ -899,7 +1092,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     }
     for (uint32_t s = lane; s < P.L.NS; s += 32) {
       uint32_t *o = P.smrec(s);
-      o[0] = NONE; o[1] = INF; o[2] = 0; o[3] = INF;
+      o[0] = NONE; o[1] = INF; o[2] = SPL ? SPLIT_NONE : 0u; o[3] = INF;
     }
     for (uint32_t j = lane; j < P.L.Scta; j += 32) P.cta(j)[C_ID] = NONE;
     for (uint32_t k = lane; k < P.L.NS * P.L.SC; k += 32) sp[P.L.o_sv + k] = 0u;
@@ -937,7 +1130,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
     const uint64_t l2_cap = l2on ? (uint64_t)prm[GTS_P_L2_BYTES] : 0ull;
     uint64_t b = INF64;  // this lane's best (effective cycle << 32 | id) over its SMs
     uint32_t bsl = 0;    // ... and its slot
-    if (!launch_ctas<EXT>(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
+    if (!launch_ctas<EXT, SPL>(g, P, C, cta_sm_row, lane, b, bsl)) status = GTS_ERR_STEP_LIMIT;
 
     while (status == GTS_OK && issued < nG) {
       // ---- next event: minimum of (effective cycle, node id) over all heads
@@ -950,7 +1143,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         if (++C.steps > C.limit) { status = GTS_ERR_STEP_LIMIT; break; }
         C.t = tn;
         if (C.next_ret <= C.t) {  // a CTA retires first: launch, then choose again
-          if (!launch_ctas<EXT>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
+          if (!launch_ctas<EXT, SPL>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
           continue;
         }
         // otherwise the minimum just found is the first issue at the new cycle
@@ -1120,7 +1313,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
       __syncwarp();
       // ---- refresh keys and summaries the issue may have changed
       if (EXT && cross_touch && deg <= 32u) {  // releases reached heads of other CTAs: their SMs and this one
-        refresh_sm<EXT>(P, sm, t, C.H, lane);
+        r_sm<EXT, SPL>(P, sm, t, C.H, lane);
         bool own = (uint32_t)lane == (sm & 31u);
         uint32_t xm = __ballot_sync(FULL, xs != NONE && xs != sm);
         uint32_t done = sm;
@@ -1130,83 +1323,84 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
           const uint32_t s2 = __shfl_sync(FULL, xs, j);
           if (s2 == done) continue;
           done = s2;
-          refresh_sm<EXT>(P, s2, t, C.H, lane);
+          r_sm<EXT, SPL>(P, s2, t, C.H, lane);
           own |= (uint32_t)lane == (s2 & 31u);
         }
         if (C.H != prevH) {  // and the SMs whose HBM heads the new horizon overtakes
           for (uint32_t s = lane; s < P.L.NS; s += 32) {
-            if (P.smrec(s)[3] < C.H) {
-              rescan_sm_lane<EXT>(P, s, t, C.H);
+            if (r_stale<SPL>(P, s, C.H)) {
+              r_rescan<EXT, SPL>(P, s, t, C.H);
               own = true;
             }
           }
         }
         if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
           const uint32_t g0 = div16(sm, P.mCsms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
-          for (uint32_t s = g0 + lane; s < g1; s += 32) rescan_sm_lane<EXT>(P, s, t, C.H);
+          for (uint32_t s = g0 + lane; s < g1; s += 32) r_rescan<EXT, SPL>(P, s, t, C.H);
           __syncwarp();
           for (uint32_t s = g0; s < g1; s++) own |= (s & 31u) == (uint32_t)lane;
         }
         __syncwarp();
-        if (own) b = lane_best(P, lane, bsl);
+        if (own) b = r_lane_best<SPL>(P, lane, C.H, bsl);
       } else if (cross_touch) {  // a node with many successors: recompute everything
-        for (uint32_t s = lane; s < P.L.NS; s += 32) rescan_sm_lane<EXT>(P, s, t, C.H);
+        for (uint32_t s = lane; s < P.L.NS; s += 32) r_rescan<EXT, SPL>(P, s, t, C.H);
         __syncwarp();
-        b = lane_best(P, lane, bsl);
+        b = r_lane_best<SPL>(P, lane, C.H, bsl);
       } else if (C.H == prevH && P.L.per <= 16u && P.L.NS <= 512u && !(EXT && P.L.nsub)) {
-        refresh_sm_owner<EXT>(P, sm, t, C.H, lane, b, bsl);
+        r_sm_owner<EXT, SPL>(P, sm, t, C.H, lane, b, bsl);
         if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
           const uint32_t g0 = div16(sm, P.mCsms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
           for (uint32_t s = g0 + lane; s < g1; s += 32)
-            if (s != sm) rescan_sm_lane<EXT>(P, s, t, C.H);
+            if (s != sm) r_rescan<EXT, SPL>(P, s, t, C.H);
           __syncwarp();
           bool mine = false;
           for (uint32_t s = g0; s < g1; s++) mine |= s != sm && (s & 31u) == (uint32_t)lane;
-          if (mine) b = lane_best(P, lane, bsl);
+          if (mine) b = r_lane_best<SPL>(P, lane, C.H, bsl);
         }
       } else {
-        refresh_sm<EXT>(P, sm, t, C.H, lane);
+        r_sm<EXT, SPL>(P, sm, t, C.H, lane);
         if (C.H != prevH && P.L.per >= 8u && !(EXT && P.L.nsub)) {
           // SMs of many slots: one SM at a time, a slot per lane
           bool own = (uint32_t)lane == (sm & 31u);
           for (uint32_t s0 = 0; s0 < P.L.NS; s0 += 32) {
             const uint32_t s = s0 + lane;
-            uint32_t xm = __ballot_sync(FULL, s < P.L.NS && s != sm && P.smrec(s)[3] < C.H);
+            uint32_t xm = __ballot_sync(FULL, s < P.L.NS && s != sm && r_stale<SPL>(P, s, C.H));
             while (xm) {
               const uint32_t s2 = s0 + __ffs(xm) - 1;
               xm &= xm - 1;
-              refresh_sm<EXT>(P, s2, t, C.H, lane);
+              r_sm<EXT, SPL>(P, s2, t, C.H, lane);
               own |= (uint32_t)lane == (s2 & 31u);
             }
           }
-          if (own) b = lane_best(P, lane, bsl);
+          if (own) b = r_lane_best<SPL>(P, lane, C.H, bsl);
         } else if (C.H != prevH) {
           // SMs whose HBM heads H overtakes change their effective cycles
           bool any = false;
           for (uint32_t s = lane; s < P.L.NS; s += 32) {
-            if (s != sm && P.smrec(s)[3] < C.H) {
-              rescan_sm_lane<EXT>(P, s, t, C.H);
+            if (s != sm && r_stale<SPL>(P, s, C.H)) {
+              r_rescan<EXT, SPL>(P, s, t, C.H);
               any = true;
             }
           }
-          if (any || (uint32_t)lane == (sm & 31u)) b = lane_best(P, lane, bsl);
+          // split records take the new H where they are read: every lane's best may move
+          if (SPL || any || (uint32_t)lane == (sm & 31u)) b = r_lane_best<SPL>(P, lane, C.H, bsl);
         } else {
-          refresh_owner(P, sm & 31u, lane, b, bsl);
+          r_owner<SPL>(P, sm & 31u, lane, C.H, b, bsl);
         }
         if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
           const uint32_t g0 = div16(sm, P.mCsms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
           for (uint32_t s = g0 + lane; s < g1; s += 32)
-            if (s != sm) rescan_sm_lane<EXT>(P, s, t, C.H);
+            if (s != sm) r_rescan<EXT, SPL>(P, s, t, C.H);
           __syncwarp();
           bool mine = false;  // this lane owns one of them
           for (uint32_t s = g0; s < g1; s++) mine |= s != sm && (s & 31u) == (uint32_t)lane;
-          if (mine) b = lane_best(P, lane, bsl);
+          if (mine) b = r_lane_best<SPL>(P, lane, C.H, bsl);
         }
       }
       __syncwarp();
       if (rem == 0u) {
         if (cend <= t) {
-          if (!launch_ctas<EXT>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
+          if (!launch_ctas<EXT, SPL>(g, P, C, cta_sm_row, lane, b, bsl)) { status = GTS_ERR_STEP_LIMIT; break; }
         } else {
           C.next_ret = min(C.next_ret, cend);
         }
@@ -1452,6 +1646,7 @@ struct gts_params {
   std::vector<uint32_t> words;  // per row: shared words, 0 if the row is invalid or too large
   std::vector<uint8_t> sched;   // per row: asks for a per-subpartition issue policy or the L2 model
   std::vector<double> cost;     // per row: estimated simulation cost (0 for invalid rows)
+  std::vector<uint8_t> wide;    // per row: SMs of 8 or more warp slots (no split SM records)
   const uint32_t *d_order = nullptr;  // processing order (gts_params_set_order), borrowed
 };
 
@@ -1854,6 +2049,7 @@ gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_p
   P->words.assign(n_points, 0u);
   P->sched.assign(n_points, 0u);
   P->cost.assign(n_points, 0.0);
+  P->wide.assign(n_points, 0);
   for (uint32_t p = 0; p < n_points; p++) {
     const int32_t *row = h.data() + (size_t)p * GTS_NPARAM;
     if (check_row(row, g->G, g->dg.class_mask) != GTS_OK) continue;
@@ -1862,6 +2058,7 @@ gts_status gts_params_upload(gts_graph *g, const int32_t *d_params, uint32_t n_p
     Layout L;
     if (make_layout(row, g->cta_off[gi + 1] - g->cta_off[gi], g->W, g->dg.class_mask, L)) {
       P->words[p] = L.words;
+      P->wide[p] = L.per >= 8u;
       // per issue the work grows slowly with the simulated SMs; the extended model costs about 3.5x
       P->cost[p] = (double)(g->node_off[gi + 1] - g->node_off[gi]) * (743.0 + L.NS) * (P->sched[p] ? 3.5 : 1.0);
     }
@@ -1902,6 +2099,7 @@ uint64_t scratch_row_bytes(const gts_graph *g) {
 struct Plan {
   uint32_t words, wpb, smem, blocks, warps;
   bool sched;  // launch the extended instance (issue policies, NoC, L2)
+  bool split;  // plain instance with split SM records (every row's SMs have fewer than 8 slots)
 };
 
 gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, uint32_t np, uint32_t flags,
@@ -1909,14 +2107,18 @@ gts_status plan_launch(const gts_graph *g, const gts_params *P, uint32_t first, 
   (void)flags;
   uint32_t words = 64;
   pl.sched = false;
+  bool wide = false;
   for (uint32_t p = first; p < first + np; p++) {
     words = std::max(words, P->words[p]);
     pl.sched = pl.sched || P->sched[p];
+    wide = wide || P->wide[p];
   }
   pl.sched = pl.sched || (g->dg.class_mask & CM_NOC) != 0u;
+  pl.split = !pl.sched && !wide;
   const uint32_t bytes = words * 4;
   pl.words = words;
-  const void *kern = pl.sched ? (const void *)k_simulate<true> : (const void *)k_simulate<false>;
+  const void *kern = pl.sched ? (const void *)k_simulate<true, false>
+                   : pl.split ? (const void *)k_simulate<false, true> : (const void *)k_simulate<false, false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)MAX_SMEM_BYTES);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   int dev = 0, sms = 0;
@@ -1990,7 +2192,7 @@ gts_status gts_simulate_batch(gts_graph *g, gts_params *P, uint32_t first_point,
       const cudaError_t em = cudaMemsetAsync(d_scratch, 0, GTS_SCRATCH_HEADER_BYTES, s);
       if (em != cudaSuccess) return cuda_fail(em, "simulate: clear the point counter");
     }
-    auto kern = pl.sched ? k_simulate<true> : k_simulate<false>;
+    auto kern = pl.sched ? k_simulate<true, false> : pl.split ? k_simulate<false, true> : k_simulate<false, false>;
     kern<<<pl.blocks, pl.wpb * 32, pl.smem, s>>>(
         g->dg, P->d_params, first_point, n_points, flags, d_start, d_finish, d_makespan, d_status,
         (flags & GTS_WANT_DIGEST) ? d_digest : nullptr, (flags & GTS_WANT_CTA_SM) ? d_cta_sm : nullptr,
