@@ -1346,7 +1346,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         for (uint32_t s = lane; s < P.L.NS; s += 32) r_rescan<EXT, SPL>(P, s, t, C.H);
         __syncwarp();
         b = r_lane_best<SPL>(P, lane, C.H, bsl);
-      } else if (C.H == prevH && P.L.per <= 16u && P.L.NS <= 512u && !(EXT && P.L.nsub)) {
+      } else if (C.H == prevH && (SPL || P.L.per <= 16u) && P.L.NS <= 512u && !(EXT && P.L.nsub)) {
         r_sm_owner<EXT, SPL>(P, sm, t, C.H, lane, b, bsl);
         if (EXT && noc_touch) {  // the group's other SMs may hold DSMEM heads keyed on that server
           const uint32_t g0 = div16(sm, P.mCsms) * P.L.csms, g1 = min(g0 + P.L.csms, P.L.NS);
@@ -1359,7 +1359,7 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
         }
       } else {
         r_sm<EXT, SPL>(P, sm, t, C.H, lane);
-        if (C.H != prevH && P.L.per >= 8u && !(EXT && P.L.nsub)) {
+        if (!SPL && C.H != prevH && P.L.per >= 8u && !(EXT && P.L.nsub)) {
           // SMs of many slots: one SM at a time, a slot per lane
           bool own = (uint32_t)lane == (sm & 31u);
           for (uint32_t s0 = 0; s0 < P.L.NS; s0 += 32) {
@@ -1373,6 +1373,19 @@ k_simulate(DevGraph g, const int32_t *__restrict__ params, uint32_t first_point,
             }
           }
           if (own) b = r_lane_best<SPL>(P, lane, C.H, bsl);
+        } else if (SPL && C.H != prevH) {
+          // split records: one pass per lane rescans its whole records that H
+          // overtook and takes its best at the new H from every record it owns
+          uint64_t nb = INF64;
+          uint32_t ns = 0;
+          for (uint32_t s = lane; s < P.L.NS; s += 32) {
+            if (s != sm && r_stale<SPL>(P, s, C.H)) r_rescan<EXT, SPL>(P, s, t, C.H);
+            uint32_t sl;
+            const uint64_t v = split_sm_best(P, s, C.H, sl);
+            if (v < nb) { nb = v; ns = sl; }
+          }
+          b = nb;
+          bsl = ns;
         } else if (C.H != prevH) {
           // SMs whose HBM heads H overtakes change their effective cycles
           bool any = false;
